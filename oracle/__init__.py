@@ -1,0 +1,128 @@
+"""fp64 CPU oracle for the extend-attention path -- TEST INFRASTRUCTURE.
+
+Only the tests, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline leg
+may import this package.  It shares no code with the CUDA library and never
+takes an input or an expected value from it.  The arithmetic lives in
+rr_oracle.c (plain loops, double precision); this file only builds it and
+marshals numpy arrays.
+
+Readings of the paper used here (it never writes the attention formula):
+* append: suffix token j of agent b lands at position P_b + j, page
+  page_table[b][pos // ps], slot pos % ps (Sec. 2, "materializes their KV
+  tensors" into the shared pool);
+* attention: causal, aligned bottom-right -- suffix row i of agent b sees all
+  P_b cached keys and the suffix keys up to and including itself (Sec. 1,
+  Sec. 2: reuse the cached prefix, compute the uncached suffix);
+* GQA: query head h reads KV head h // (Hq // Hkv).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SO = os.path.join(_HERE, "librr_oracle.so")
+
+OK, BAD_ARG, BAD_PAGE, NO_MEM = 0, 1, 2, 3
+
+
+def build(verbose: bool = False) -> None:
+    cmd = ["gcc", "-O2", "-fPIC", "-shared", "-pthread", "-std=c11",
+           os.path.join(_HERE, "rr_oracle.c"), "-o", _SO, "-lm"]
+    if verbose:
+        print(" ".join(cmd))
+    subprocess.run(cmd, check=True)
+
+
+_lib = None
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        if not os.path.exists(_SO):
+            build()
+        L = ctypes.CDLL(_SO)
+        vp, i32, i64, f64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_double
+        L.oracle_kv_append.restype = ctypes.c_int
+        L.oracle_kv_append.argtypes = [vp, vp, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, i64]
+        L.oracle_extend_attention.restype = ctypes.c_int
+        L.oracle_extend_attention.argtypes = [vp, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, i64, f64,
+                                              vp, vp, vp, i32]
+        L.oracle_attention_rows.restype = ctypes.c_int
+        L.oracle_attention_rows.argtypes = [vp, vp, i64, vp, vp, i64, i32, i32, f64, vp, vp, vp, i32]
+        _lib = L
+    return _lib
+
+
+class OracleError(RuntimeError):
+    pass
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+def _p(a):
+    return a.ctypes.data if a is not None else None
+
+
+def _threads(n):
+    return n if n and n > 0 else (os.cpu_count() or 1)
+
+
+def kv_append(k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens):
+    """Returns new (k_pool, v_pool) uint16 arrays with the suffix rows written (inputs are not modified)."""
+    k_new, v_new = _c(k_new, np.uint16), _c(v_new, np.uint16)
+    kp, vp = np.array(k_pool, dtype=np.uint16, copy=True), np.array(v_pool, dtype=np.uint16, copy=True)
+    pt, pl, sl = _c(page_table, np.int32), _c(prefix_lens, np.int32), _c(suffix_lens, np.int32)
+    num_pages, ps, Hkv, D = kp.shape
+    rc = lib().oracle_kv_append(_p(k_new), _p(v_new), _p(kp), _p(vp), _p(pt), _p(pl), _p(sl), len(pl), Hkv, D,
+                                ps, pt.shape[1], num_pages)
+    if rc:
+        raise OracleError(f"oracle_kv_append: {rc}")
+    return kp, vp
+
+
+def extend_attention(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, scale=None, nthreads=0,
+                     with_stats=False):
+    """out [T, Hq, D] float64 (and lse, wsum [T, Hq] if with_stats) from bf16-bit inputs."""
+    q = _c(q, np.uint16)
+    kp, vp = _c(k_pool, np.uint16), _c(v_pool, np.uint16)
+    pt, pl, sl = _c(page_table, np.int32), _c(prefix_lens, np.int32), _c(suffix_lens, np.int32)
+    T, Hq, D = q.shape
+    num_pages, ps, Hkv, D2 = kp.shape
+    assert D2 == D and int(sl.sum()) == T
+    if scale is None:
+        scale = 1.0 / np.sqrt(D)
+    out = np.zeros((T, Hq, D), dtype=np.float64)
+    lse = np.zeros((T, Hq), dtype=np.float64) if with_stats else None
+    wsum = np.zeros((T, Hq), dtype=np.float64) if with_stats else None
+    rc = lib().oracle_extend_attention(_p(q), _p(kp), _p(vp), _p(pt), _p(pl), _p(sl), len(pl), Hq, Hkv, D, ps,
+                                       pt.shape[1], num_pages, float(scale), _p(out), _p(lse), _p(wsum),
+                                       _threads(nthreads))
+    if rc:
+        raise OracleError(f"oracle_extend_attention: {rc}")
+    return (out, lse, wsum) if with_stats else out
+
+
+def attention_rows(q_rows, positions, K, V, scale, nthreads=0, with_stats=False):
+    """Selected rows of one agent / one KV group over its logical K, V ([n_keys, D] bf16 bits).
+
+    q_rows: [n, G, D] bf16 bits; positions: [n] absolute positions.  Returns out [n, G, D] float64.
+    """
+    q_rows = _c(q_rows, np.uint16)
+    positions = _c(positions, np.int64)
+    K, V = _c(K, np.uint16), _c(V, np.uint16)
+    n, G, D = q_rows.shape
+    out = np.zeros((n, G, D), dtype=np.float64)
+    lse = np.zeros((n, G), dtype=np.float64) if with_stats else None
+    wsum = np.zeros((n, G), dtype=np.float64) if with_stats else None
+    rc = lib().oracle_attention_rows(_p(q_rows), _p(positions), n, _p(K), _p(V), K.shape[0], G, D, float(scale),
+                                     _p(out), _p(lse), _p(wsum), _threads(nthreads))
+    if rc:
+        raise OracleError(f"oracle_attention_rows: {rc}")
+    return (out, lse, wsum) if with_stats else out
