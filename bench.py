@@ -1,0 +1,401 @@
+"""Benchmark of one extend step on GB300: KV append + extend attention over a paged KV pool.
+
+A step is the whole hot path for one batch of returning agents: on-device
+schedule, KV append of every uncached suffix token into its pool slot, and
+extend attention of every suffix row over its agent's cached prefix and
+suffix.  Default workload: the Llama-3-8B attention shape (32 agents, 32 query
+/ 8 KV heads, d128, page size 16, cached prefixes U[8k,32k] ending on 512-token
+chunk boundaries, suffixes U[256,2048], seeded page placement), synthetic
+N(0,1) bf16 data.
+
+Prints one JSON line.  `value` is the algorithmic attention TFLOP/s of the
+whole step (append included) with inputs resident in HBM; `e2e` is the same
+metric through the public API with host (pinned) inputs and output, copies
+inside the timed region.  The roofline object is for the dominant kernel
+(extend attention, tensor-core bound).  `--impl reference` times the fp64 CPU
+oracle on the host cores instead, on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "extend-attn TFLOP/s & uncached suffix tokens/s on 1 GB300; % of roofline"
+NOMINAL_BF16_TFLOPS = 2250.0
+NOMINAL_HBM_GBS = 8000.0
+
+
+def attn_flops(wl) -> float:
+    """Algorithmic flops: 4 * D * Hq * sum_b (S_b * P_b + S_b (S_b + 1) / 2) (masked work not counted)."""
+    P = wl.prefix_lens.astype(np.float64)
+    S = wl.suffix_lens.astype(np.float64)
+    return float(4.0 * wl.D * wl.Hq * np.sum(S * P + S * (S + 1) / 2))
+
+
+def attn_bytes(wl) -> float:
+    """Algorithmic bytes: each agent's K and V once per KV head, q in, out out, lens and page table."""
+    kv = float(np.sum((wl.prefix_lens.astype(np.float64) + wl.suffix_lens) * wl.Hkv * wl.D * 2 * 2))
+    qo = 2.0 * wl.T * wl.Hq * wl.D * 2
+    meta = wl.page_table.size * 4 + 2 * wl.B * 4
+    return kv + qo + meta
+
+
+def append_bytes(wl) -> float:
+    return 4.0 * wl.T * wl.Hkv * wl.D * 2
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for f in ("extend_attn.cu", "ptx.cuh", "rr_internal.h"):
+        with open(os.path.join(ROOT, "paper_2609_32278_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return dict(hbm=p["hbm_gbs"], bf16=p["bf16_tflops"], bf16_sus=p["bf16_tflops_sustained"], src="measured")
+    except Exception:
+        return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+        sm, smax, reasons = [], None, set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax = float(parts[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": smax, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if args.impl == "ours" else "gloo"
+        if backend == "nccl":
+            import torch
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend=backend)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x, world, device=None):
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device if device is not None else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def cpu_oracle_sample(wl, flop_budget: float, seed: int):
+    """Time the fp64 oracle on sampled suffix rows (generation of K/V is not timed)."""
+    import oracle
+    import synth
+    rng = np.random.default_rng(seed)
+    live = [b for b in range(wl.B) if wl.suffix_lens[b] > 0]
+    per_row = lambda b, i: 4.0 * wl.D * wl.Hq * (int(wl.prefix_lens[b]) + i + 1)
+    picks, spent = {}, 0.0
+    while spent < flop_budget:
+        b = int(rng.choice(live))
+        i = int(rng.integers(0, int(wl.suffix_lens[b])))
+        picks.setdefault(b, set()).add(i)
+        spent += per_row(b, i)
+    threads = os.cpu_count() or 1
+    total_t, total_f, rows = 0.0, 0.0, 0
+    for b, rs in picks.items():
+        rs = np.array(sorted(rs), dtype=np.int64)
+        pos = int(wl.prefix_lens[b]) + rs
+        L = int(pos.max()) + 1
+        qr = synth.q_rows(wl, b, pos)
+        for g in range(wl.Hkv):
+            K, V = synth.agent_kv(wl, b, L, g)
+            t0 = time.perf_counter()
+            oracle.attention_rows(qr[:, g * wl.G:(g + 1) * wl.G], pos, K, V, 1.0 / math.sqrt(wl.D), threads)
+            total_t += time.perf_counter() - t0
+        total_f += sum(per_row(b, int(i)) for i in rs)
+        rows += len(rs)
+    return total_f, total_t, rows, threads
+
+
+def run_reference(args, world, rank):
+    import synth
+    if rank != 0:
+        return 0
+    wl = synth.config(args.config, seed=0)
+    budget = args.ref_flops
+    for _ in range(args.warmup):
+        cpu_oracle_sample(wl, budget, seed=1000)
+    fl, tm, rows, threads = 0.0, 0.0, 0, 1
+    for k in range(args.steps):
+        f, t, r, threads = cpu_oracle_sample(wl, budget, seed=k)
+        fl += f
+        tm += t
+        rows += r
+    value = fl / tm / 1e12
+    tok_per_s = rows / tm
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": tm / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": args.config, "B": wl.B, "Hq": wl.Hq, "Hkv": wl.Hkv, "D": wl.D, "page_size": wl.ps,
+                   "uncached_tokens": wl.T},
+        "uncached_suffix_tokens_per_s": tok_per_s,
+        "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": threads, "kind": "oracle",
+                         "sample": f"{rows} seeded suffix rows (all heads) over {args.steps} steps, "
+                                   f"~{budget:.1e} flop each; fp64 oracle, K/V generation not timed"},
+        "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def load_traffic(src_hash):
+    """DRAM bytes per attention launch from the committed ncu summary, if it was taken on this kernel source."""
+    path = os.path.join(ROOT, "profiles", "extend_attn_traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+    except Exception:
+        return None, None
+    if rec.get("kernel_source_hash") != src_hash:
+        return None, rec
+    return rec, rec
+
+
+def run_ours(args, world, rank, local):
+    import torch
+    import synth
+    import paper_2609_32278_gb300 as rr
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    free = torch.cuda.mem_get_info(dev)[0]
+    wl = synth.config(args.config, seed=rank, free_hbm_bytes=free if args.config == "c4_coding" else None)
+    g = synth.gpu_tensors(wl, dev)
+    st = torch.cuda.current_stream(dev)
+    F = attn_flops(wl)
+    peaks = load_peaks()
+
+    def step():
+        rr.kv_append(g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                     g["suffix_lens"])
+        return rr.extend_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                                   g["suffix_lens"], out=g["out"])
+
+    g["out"] = torch.empty_like(g["q"])
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize(dev)
+    code = rr.device_error()
+    if code:
+        raise RuntimeError(f"device error {code} during warm-up")
+
+    # ---- device-timed steps (inputs resident in HBM; working set > L2)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+           torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(st)
+    for k in range(args.steps):
+        e0, e1, e2 = ev[k]
+        e0.record(st)
+        rr.kv_append(g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                     g["suffix_lens"])
+        e1.record(st)
+        rr.extend_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"], g["suffix_lens"],
+                            out=g["out"])
+        e2.record(st)
+    t_end.record(st)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clk = clocks.stop()
+    code = rr.device_error()
+    if code:
+        raise RuntimeError(f"device error {code} in the timed region")
+    total_ms = t_start.elapsed_time(t_end)
+    total_ms = max_over_ranks(total_ms, world, dev)
+    ms_step = total_ms / args.steps
+    attn_ms = statistics.mean(ev[k][1].elapsed_time(ev[k][2]) for k in range(args.steps))
+    app_ms = statistics.mean(ev[k][0].elapsed_time(ev[k][1]) for k in range(args.steps))
+    value = world * F / (ms_step * 1e-3) / 1e12
+    tok_s = world * wl.T / (ms_step * 1e-3)
+
+    # ---- end to end through the public API: pinned host inputs -> device -> step -> host output
+    host = {k: g[k].cpu().pin_memory() for k in ("q", "k_new", "v_new", "page_table", "prefix_lens", "suffix_lens")}
+    out_h = torch.empty(g["q"].shape, dtype=torch.bfloat16).pin_memory()
+    dev_in = {k: torch.empty_like(g[k]) for k in host}
+    h2d = sum(v.numel() * v.element_size() for v in host.values())
+    d2h = out_h.numel() * out_h.element_size()
+
+    def e2e_step():
+        for k, v in host.items():
+            dev_in[k].copy_(v, non_blocking=True)
+        rr.kv_append(dev_in["k_new"], dev_in["v_new"], g["k_pool"], g["v_pool"], dev_in["page_table"],
+                     dev_in["prefix_lens"], dev_in["suffix_lens"])
+        rr.extend_attention(dev_in["q"], g["k_pool"], g["v_pool"], dev_in["page_table"], dev_in["prefix_lens"],
+                            dev_in["suffix_lens"], out=g["out"])
+        out_h.copy_(g["out"], non_blocking=True)
+
+    for _ in range(args.warmup):
+        e2e_step()
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    s0 = torch.cuda.Event(enable_timing=True)
+    s1 = torch.cuda.Event(enable_timing=True)
+    s0.record(st)
+    for _ in range(args.steps):
+        e2e_step()
+    s1.record(st)
+    torch.cuda.synchronize(dev)
+    e2e_ms = max_over_ranks(s0.elapsed_time(s1) / args.steps, world, dev)
+    if rr.device_error():
+        raise RuntimeError("device error in the end-to-end region")
+
+    achieved = F / (attn_ms * 1e-3) / 1e12
+    src_hash = kernel_source_hash()
+    traffic_rec, _ = load_traffic(src_hash)
+    traffic = None
+    if traffic_rec is not None and traffic_rec.get("workload") == args.config:
+        traffic = traffic_rec.get("dram_bytes_per_launch")
+    roof = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
+            "frac": achieved / peaks["bf16_sus"], "traffic": traffic,
+            "peak_kind": f"{peaks['src']} bf16 dense, sustained (kernel timed inside a seconds-long loop)",
+            "frac_of_burst": achieved / peaks["bf16"], "frac_of_nominal": achieved / NOMINAL_BF16_TFLOPS,
+            "kernel": "extend_attn_kernel<128,2>" if wl.D == 128 else "extend_attn_kernel<64,4>",
+            "algorithmic_bytes": attn_bytes(wl), "algorithmic_flops": F,
+            "bytes_bound_frac": attn_bytes(wl) / (attn_ms * 1e-3) / 1e9 / peaks["hbm"],
+            "kernel_source_hash": src_hash}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": args.config, "B": wl.B, "Hq": wl.Hq, "Hkv": wl.Hkv, "D": wl.D, "page_size": wl.ps,
+                   "uncached_tokens": wl.T, "kv_tokens": int((wl.prefix_lens + wl.suffix_lens).sum()),
+                   "num_pages": wl.num_pages, "l2": "inputs larger than L2 (KV working set "
+                   f"{attn_bytes(wl) / 1e9:.1f} GB > 129 MB)", "parallelism": f"replicas x{world}"},
+        "uncached_suffix_tokens_per_s": tok_s,
+        "attention_ms": attn_ms, "kv_append_ms": app_ms,
+        "kv_append_gbs": append_bytes(wl) / (app_ms * 1e-3) / 1e9,
+        "roofline": roof,
+        "e2e": {"value": world * F / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+        "gpu_launches": 4 * args.steps,
+        "clocks": clk,
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        f, t, rows, threads = cpu_oracle_sample(wl, args.baseline_flops, seed=7)
+        line["cpu_baseline"] = {"value": f / t / 1e12, "unit": "TFLOP/s", "cores": threads, "kind": "oracle",
+                                "sample": f"{rows} seeded suffix rows (all {wl.Hq} heads) of {args.config}, "
+                                          f"{f:.2e} flop; fp64 oracle; K/V generation not timed"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--config", default="c2_llama3_8b")
+    ap.add_argument("--ref-flops", type=float, default=1e10, help="oracle flops per reference-arm step")
+    ap.add_argument("--baseline-flops", type=float, default=6e10, help="oracle flops of the cpu_baseline sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    world, rank, local = dist_setup(args)
+    try:
+        if args.impl == "reference":
+            return run_reference(args, world, rank)
+        return run_ours(args, world, rank, local)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    sys.exit(main())

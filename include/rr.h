@@ -1,0 +1,145 @@
+/*
+ * rr.h -- C ABI of librr.so, the GB300 (sm_103a) extend-attention library.
+ *
+ * The path it implements is the "extend" prefill of agents that return to a
+ * prefix-cached serving engine (RR-Evict, Sec. 1 and Sec. 2: the engine reuses
+ * the cached KV tensors of an agent's surviving prefix and computes only the
+ * uncached suffix; the suffix's new KV tensors are materialised into the
+ * shared, paged KV pool, Sec. 2).  Which prefix survives is decided by the
+ * eviction policy (round-robin tail-chunk eviction, Algorithm 1, versus LRU,
+ * Sec. 3.1-3.2); the kernels take the resulting per-agent lengths as input.
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ *  * B agents; Hq query heads; Hkv KV heads, G = Hq / Hkv query heads per KV
+ *    head (query head h reads KV head h / G); D head dim; ps tokens per page.
+ *  * Agent b has a cached prefix of P_b = prefix_lens[b] tokens and an
+ *    uncached suffix of S_b = suffix_lens[b] tokens.  Suffix token j of agent
+ *    b has absolute position P_b + j.  Agents' suffix rows are packed in agent
+ *    order: agent b owns rows cu_b .. cu_b + S_b - 1 of q / out / k_new /
+ *    v_new, cu_b = S_0 + ... + S_{b-1};  T = sum of S_b = dims->total_tokens.
+ *  * Layouts (row-major, contiguous, bf16 = IEEE bfloat16):
+ *        q, out        [T, Hq, D]                 bf16
+ *        k_new, v_new  [T, Hkv, D]                bf16
+ *        k_pool,v_pool [num_pages, ps, Hkv, D]    bf16
+ *        page_table    [B, max_pages]             int32, physical page of
+ *                      logical page i of agent b (position i*ps .. i*ps+ps-1);
+ *                      entries past ceil((P_b+S_b)/ps) are never read.
+ *        prefix_lens, suffix_lens  [B]            int32
+ *  * Memory: every pointer is a DEVICE pointer on the current device, owned
+ *    by the caller; q/out/k_new/v_new/pools must be 16-byte aligned.  The
+ *    library keeps one growable per-device workspace (schedule, error word),
+ *    allocated on first use and freed by rr_shutdown().
+ *  * Streams: calls enqueue work on `stream` and return without waiting; the
+ *    lens stay on the device (the schedule is built on the device).
+ *  * Errors: a call returns RR_OK or an RR_ERR_* code and never aborts; the
+ *    message of the last failure on the calling thread is rr_last_error().
+ *    Problems only the device can see (lens inconsistent with total_tokens,
+ *    a page id outside the pool, a wait that timed out) are recorded in a
+ *    device error word instead of faulting: read it with rr_get_device_error.
+ */
+#ifndef RR_H_
+#define RR_H_
+
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define RR_OK 0
+#define RR_ERR_INVALID_ARG 1   /* null pointer, negative size, misaligned pointer */
+#define RR_ERR_UNSUPPORTED 2   /* D not 64/128, G not in {1,2,4,8,16}, ps not in {16,32,64,128} */
+#define RR_ERR_CUDA 3          /* a CUDA runtime/driver call failed */
+#define RR_ERR_TIMEOUT 4       /* device: a bounded pipeline wait gave up (the kernel returned early) */
+#define RR_ERR_OOB 5           /* device or host: a page id outside [0, num_pages) */
+#define RR_ERR_LENS 6          /* device: negative length, P_b+S_b > max_pages*ps, or sum S_b != T */
+#define RR_ERR_OVERLAP 7       /* host validation: a suffix page is shared with another agent or a prefix */
+
+/* Sizes of one call.  All counts are in elements or tokens, not bytes. */
+typedef struct rr_dims {
+    int32_t batch;         /* B, number of agents (>= 0) */
+    int32_t num_q_heads;   /* Hq */
+    int32_t num_kv_heads;  /* Hkv; Hq % Hkv == 0 */
+    int32_t head_dim;      /* D: 64 or 128 */
+    int32_t page_size;     /* ps: tokens per page */
+    int32_t max_pages;     /* columns of page_table */
+    int64_t num_pages;     /* pages in EACH of k_pool and v_pool */
+    int64_t total_tokens;  /* T = sum of suffix_lens (rows of q/out/k_new/v_new) */
+} rr_dims;
+
+/*
+ * rr_kv_append -- write the uncached suffix's K/V into the pool (Sec. 2: the
+ * prefill "materializes" the KV tensors of the tokens it processes; they go
+ * into the shared pool so later turns can reuse them, Sec. 2 / Sec. 3.1).
+ *
+ * For every agent b and j < S_b, with pos = P_b + j:
+ *     k_pool[page_table[b][pos / ps], pos % ps, :, :] = k_new[cu_b + j, :, :]
+ *     v_pool[ ... same slot ... ]                      = v_new[cu_b + j, :, :]
+ * Bytes are copied unchanged; no other pool byte is written.  The pages that
+ * hold suffix positions must be distinct across agents (rr_validate_page_table
+ * checks this on the host); pages shared between agents (a common system
+ * prompt) are only ever read.  A page id outside the pool is skipped and
+ * recorded as RR_ERR_OOB in the device error word.
+ */
+int rr_kv_append(const void* k_new, const void* v_new, void* k_pool, void* v_pool, const int32_t* page_table,
+                 const int32_t* prefix_lens, const int32_t* suffix_lens, const rr_dims* dims,
+                 cudaStream_t stream);
+
+/*
+ * rr_extend_attention -- attention of every uncached suffix row over the
+ * agent's cached prefix and its own suffix (Sec. 1 and Sec. 2: the returning
+ * agent reuses its surviving prefix and prefills the missing suffix).
+ *
+ * For agent b, suffix row i, query head h, g = h / G, p = P_b + i:
+ *     s_j = scale * <q[cu_b+i, h, :], K_j>      for keys j = 0 .. p
+ *     out[cu_b+i, h, :] = sum_j softmax(s)_j V_j
+ * where K_j, V_j are position j of agent b, KV head g, read from
+ * k_pool/v_pool through page_table.  The row sees the whole prefix and the
+ * suffix up to and including itself (causal mask aligned bottom-right).
+ * softmax_scale <= 0 selects 1/sqrt(D).  bf16 inputs, fp32 accumulation and
+ * softmax, bf16 output rounded to nearest even.
+ *
+ * The suffix's K/V must already be in the pool: call rr_kv_append first on
+ * the same stream.  Pool slots past an agent's last position are never read
+ * into the result, whatever they contain.  The output is a deterministic
+ * function of the logical inputs: it does not depend on the physical page
+ * placement or on the order in which agents are listed.
+ */
+int rr_extend_attention(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
+                        const int32_t* prefix_lens, const int32_t* suffix_lens, void* out, const rr_dims* dims,
+                        float softmax_scale, cudaStream_t stream);
+
+/*
+ * rr_validate_page_table -- HOST-side check of a page table before use
+ * (host arrays, not device).  Returns RR_OK, RR_ERR_LENS (bad lengths),
+ * RR_ERR_OOB (a page an agent uses is outside [0, num_pages)) or
+ * RR_ERR_OVERLAP (a page holding suffix positions of one agent is used by
+ * any other agent, or by the same agent twice).  Reads only; allocates a
+ * bitmap of num_pages bits on the host.
+ */
+int rr_validate_page_table(const int32_t* page_table, const int32_t* prefix_lens, const int32_t* suffix_lens,
+                           const rr_dims* dims);
+
+/*
+ * rr_get_device_error -- synchronise `stream`, return the device error word
+ * of the current device (RR_OK or an RR_ERR_* code recorded by a kernel since
+ * the last read) and reset it to RR_OK.
+ */
+int rr_get_device_error(cudaStream_t stream);
+
+/* Message of the last failing call on this thread ("" if none). */
+const char* rr_last_error(void);
+
+/* Library version string. */
+const char* rr_version(void);
+
+/* Free the per-device workspaces (synchronises each device that has one). */
+void rr_shutdown(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RR_H_ */

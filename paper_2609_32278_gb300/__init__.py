@@ -1,0 +1,192 @@
+"""GB300 extend attention over a paged KV pool -- Python binding of librr.so.
+
+Two calls make one extend step for a batch of returning agents (RR-Evict,
+Sec. 1-2: reuse each agent's surviving cached prefix, prefill its uncached
+suffix):
+
+    kv_append(k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens)
+    out = extend_attention(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens)
+
+This module only marshals torch tensors into the C ABI of include/rr.h; every
+step of the computation runs in the CUDA kernels of librr.so.  There is no
+fallback: if the library is missing or a call fails, an exception is raised.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SO = os.path.join(_HERE, "librr.so")
+
+RR_OK = 0
+RR_ERR_INVALID_ARG = 1
+RR_ERR_UNSUPPORTED = 2
+RR_ERR_CUDA = 3
+RR_ERR_TIMEOUT = 4
+RR_ERR_OOB = 5
+RR_ERR_LENS = 6
+RR_ERR_OVERLAP = 7
+
+# Every symbol include/rr.h declares.
+EXPORTS = ("rr_kv_append", "rr_extend_attention", "rr_validate_page_table", "rr_get_device_error",
+           "rr_last_error", "rr_version", "rr_shutdown")
+
+
+class RRError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"rr error {code}: {msg}")
+        self.code = code
+
+
+class Dims(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("num_q_heads", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("page_size", ctypes.c_int32), ("max_pages", ctypes.c_int32),
+                ("num_pages", ctypes.c_int64), ("total_tokens", ctypes.c_int64)]
+
+
+_lib = None
+
+
+def build(verbose: bool = False) -> str:
+    from . import native_build
+    return native_build.build(verbose=verbose)
+
+
+def lib():
+    """The loaded librr.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(_SO):
+            raise RuntimeError(f"{_SO} not found: build it with __graft_entry__.build() "
+                               "(there is no fallback implementation)")
+        L = ctypes.CDLL(_SO)
+        vp = ctypes.c_void_p
+        dp = ctypes.POINTER(Dims)
+        L.rr_kv_append.restype = ctypes.c_int
+        L.rr_kv_append.argtypes = [vp, vp, vp, vp, vp, vp, vp, dp, vp]
+        L.rr_extend_attention.restype = ctypes.c_int
+        L.rr_extend_attention.argtypes = [vp, vp, vp, vp, vp, vp, vp, dp, ctypes.c_float, vp]
+        L.rr_validate_page_table.restype = ctypes.c_int
+        L.rr_validate_page_table.argtypes = [vp, vp, vp, dp]
+        L.rr_get_device_error.restype = ctypes.c_int
+        L.rr_get_device_error.argtypes = [vp]
+        L.rr_last_error.restype = ctypes.c_char_p
+        L.rr_last_error.argtypes = []
+        L.rr_version.restype = ctypes.c_char_p
+        L.rr_version.argtypes = []
+        L.rr_shutdown.restype = None
+        L.rr_shutdown.argtypes = []
+        _lib = L
+    return _lib
+
+
+def _check(rc: int) -> None:
+    if rc != RR_OK:
+        raise RRError(rc, lib().rr_last_error().decode(errors="replace"))
+
+
+def _stream_ptr(stream, device):
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream(device)
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _need(t, name, dtype, ndim):
+    import torch
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if t.dim() != ndim:
+        raise ValueError(f"{name} must have {ndim} dims, got {tuple(t.shape)}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+
+
+def make_dims(B, Hq, Hkv, D, ps, max_pages, num_pages, T) -> Dims:
+    return Dims(int(B), int(Hq), int(Hkv), int(D), int(ps), int(max_pages), int(num_pages), int(T))
+
+
+def kv_append(k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens, stream=None) -> None:
+    """Write suffix K/V rows into their pool slots (see rr_kv_append in include/rr.h)."""
+    import torch
+    _need(k_new, "k_new", torch.bfloat16, 3)
+    _need(v_new, "v_new", torch.bfloat16, 3)
+    _need(k_pool, "k_pool", torch.bfloat16, 4)
+    _need(v_pool, "v_pool", torch.bfloat16, 4)
+    _need(page_table, "page_table", torch.int32, 2)
+    _need(prefix_lens, "prefix_lens", torch.int32, 1)
+    _need(suffix_lens, "suffix_lens", torch.int32, 1)
+    T, Hkv, D = k_new.shape
+    num_pages, ps, Hkv2, D2 = k_pool.shape
+    if v_new.shape != k_new.shape or v_pool.shape != k_pool.shape or (Hkv2, D2) != (Hkv, D):
+        raise ValueError("k/v shapes disagree")
+    B = prefix_lens.shape[0]
+    if suffix_lens.shape[0] != B or page_table.shape[0] != B:
+        raise ValueError("lens / page_table batch sizes disagree")
+    dims = make_dims(B, Hkv, Hkv, D, ps, page_table.shape[1], num_pages, T)
+    _check(lib().rr_kv_append(k_new.data_ptr(), v_new.data_ptr(), k_pool.data_ptr(), v_pool.data_ptr(),
+                              page_table.data_ptr(), prefix_lens.data_ptr(), suffix_lens.data_ptr(),
+                              ctypes.byref(dims), _stream_ptr(stream, k_new.device)))
+
+
+def extend_attention(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, out=None,
+                     softmax_scale: float = 0.0, stream=None):
+    """Extend attention of every suffix row over its agent's prefix + suffix (rr_extend_attention)."""
+    import torch
+    _need(q, "q", torch.bfloat16, 3)
+    _need(k_pool, "k_pool", torch.bfloat16, 4)
+    _need(v_pool, "v_pool", torch.bfloat16, 4)
+    _need(page_table, "page_table", torch.int32, 2)
+    _need(prefix_lens, "prefix_lens", torch.int32, 1)
+    _need(suffix_lens, "suffix_lens", torch.int32, 1)
+    T, Hq, D = q.shape
+    num_pages, ps, Hkv, D2 = k_pool.shape
+    if v_pool.shape != k_pool.shape or D2 != D:
+        raise ValueError("q / pool shapes disagree")
+    B = prefix_lens.shape[0]
+    if suffix_lens.shape[0] != B or page_table.shape[0] != B:
+        raise ValueError("lens / page_table batch sizes disagree")
+    if out is None:
+        out = torch.empty_like(q)
+    else:
+        _need(out, "out", torch.bfloat16, 3)
+        if out.shape != q.shape:
+            raise ValueError("out must have q's shape")
+    dims = make_dims(B, Hq, Hkv, D, ps, page_table.shape[1], num_pages, T)
+    _check(lib().rr_extend_attention(q.data_ptr(), k_pool.data_ptr(), v_pool.data_ptr(), page_table.data_ptr(),
+                                     prefix_lens.data_ptr(), suffix_lens.data_ptr(), out.data_ptr(),
+                                     ctypes.byref(dims), float(softmax_scale), _stream_ptr(stream, q.device)))
+    return out
+
+
+def device_error(stream=None, device=None) -> int:
+    """Synchronise the stream and return (and clear) the device error word."""
+    import torch
+    dev = device if device is not None else torch.device("cuda", torch.cuda.current_device())
+    return int(lib().rr_get_device_error(_stream_ptr(stream, dev)))
+
+
+def validate_page_table(page_table, prefix_lens, suffix_lens, num_pages: int, page_size: int,
+                        total_tokens: Optional[int] = None) -> int:
+    """Host-side page-table check (numpy int32 arrays); returns an RR_* code, never raises on bad tables."""
+    import numpy as np
+    pt = np.ascontiguousarray(page_table, dtype=np.int32)
+    pl = np.ascontiguousarray(prefix_lens, dtype=np.int32)
+    sl = np.ascontiguousarray(suffix_lens, dtype=np.int32)
+    T = int(sl.sum()) if total_tokens is None else int(total_tokens)
+    dims = make_dims(len(pl), 1, 1, 64, page_size, pt.shape[1] if pt.ndim == 2 else 0, num_pages, T)
+    return int(lib().rr_validate_page_table(pt.ctypes.data, pl.ctypes.data, sl.ctypes.data, ctypes.byref(dims)))
+
+
+def last_error() -> str:
+    return lib().rr_last_error().decode(errors="replace")
+
+
+def version() -> str:
+    return lib().rr_version().decode()

@@ -1,0 +1,505 @@
+// extend_attn.cu -- paged-KV extend attention for sm_103a (tcgen05 + TMEM + TMA).
+//
+// What it computes (Sec. 1, Sec. 2): every uncached suffix row of a returning
+// agent attends causally to the agent's cached prefix and to the suffix up to
+// itself; K/V come from the shared paged pool through the agent's page table.
+//
+//   out[cu_b+i, h, :] = softmax_j( scale * q[cu_b+i, h, :] . K_j ) V_j,  j = 0 .. P_b + i
+//
+// Design (one persistent CTA per SM, 10 warps):
+//   * work unit = (agent b, KV head g, kNQ = 2 consecutive Q tiles).  A Q tile
+//     packs 128/G suffix tokens x the G query heads that share KV head g into
+//     128 rows (GQA packing), so each K/V tile is loaded once for the whole
+//     group and feeds M = 128 MMAs.  Units come from the on-device schedule,
+//     most expensive first, dealt to CTAs in a snake order.
+//   * warp 8, TMA producer: Q tiles (one 3-D box per 64-column chunk) and, per
+//     128-key KV tile, one 2-D box per page and chunk -- the page gather.  Pages
+//     past the agent's keys are requested at a row past the pool, which TMA
+//     fills with zeros; slots of the agent's last page that lie past its last
+//     position are cleared in shared memory before the MMA may read V.
+//   * warp 9, MMA issuer (one thread): S_q = Q_q K^T  (SS, both operands
+//     K-major, 128B swizzle) into TMEM, and O_q += P_q V (TS: P read from TMEM,
+//     V from shared memory as an MN-major operand).  Issue order per KV tile j:
+//     PV_0(j), S_0(j+1), PV_1(j), S_1(j+1): the tensor core works on one Q
+//     tile while the softmax warpgroup of the other runs.
+//   * warps 0-3 / 4-7, softmax warpgroups for Q tile 0 / 1: thread r owns row
+//     r (= TMEM lane r).  It loads its S row from TMEM, applies the causal mask
+//     on the tiles that need it, keeps a running max in log2 units and rescales
+//     O only when the max grew by more than 2^8 (the stale max keeps every
+//     probability <= 256, far inside bf16/fp32 range), writes P as bf16 back
+//     over its S columns, and at the end of the unit normalises O and stores it.
+//   TMEM: S_0 cols 0-127, S_1 128-255, O_0 256.., O_1 256+D.. (512 allocated).
+//   Shared memory (D=128): Q 2 x 32 KiB, K and V 2 stages x 32 KiB each.
+//
+// Ordering facts the pipeline relies on: tcgen05.mma operations issued by one
+// thread execute in order, and tcgen05.commit arrives only after every earlier
+// MMA of that thread finished; so when S_q(j) is complete, PV_q(j-1) is too,
+// and the softmax may rescale O_q without another wait.
+//
+// Every wait is bounded (clock64 budget); a wait that runs out sets the
+// device error word to RR_ERR_TIMEOUT and a shared abort flag, every role
+// leaves its loop, in-flight copies and MMAs are drained, TMEM is freed and
+// the kernel returns.  No trap, no unbounded spin.
+#include <cuda_bf16.h>
+
+#include "ptx.cuh"
+#include "rr_internal.h"
+
+namespace rr {
+
+namespace {
+
+constexpr int kThreads = 320;
+constexpr int kWarpProducer = 8;
+constexpr int kWarpMMA = 9;
+constexpr long long kWaitLimitCycles = 1ll << 33;  // ~4 s at 2 GHz
+
+template <int D, int NS>
+struct Cfg {
+    static constexpr int kChunks = D / 64;                 // 128-byte (64 x bf16) column chunks
+    static constexpr int kChunkBytes = kBM * 128;          // one chunk of a 128-row tile: 16 KiB
+    static constexpr int kQTileBytes = kBM * D * 2;
+    static constexpr int kKVTileBytes = kBN * D * 2;
+    static constexpr int kOffQ = 0;
+    static constexpr int kOffK = kOffQ + kNQ * kQTileBytes;
+    static constexpr int kOffV = kOffK + NS * kKVTileBytes;
+    static constexpr int kOffBar = kOffV + NS * kKVTileBytes;
+    // barrier indices
+    static constexpr int kQFull = 0, kQEmpty = 1;
+    static constexpr int kKFull = 2, kKEmpty = 2 + NS, kVFull = 2 + 2 * NS, kVEmpty = 2 + 3 * NS;
+    static constexpr int kSFull = 2 + 4 * NS, kPFull = kSFull + kNQ, kOFinal = kPFull + kNQ;
+    static constexpr int kVTmp = kOFinal + kNQ, kDrain = kVTmp + 1;
+    static constexpr int kNumBars = kDrain + 1;
+    static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // u32 TMEM base, i32 abort flag
+    static constexpr int kSmemBytes = kOffMisc + 16 + 1024;  // + slack to align the base to 1 KiB
+    static_assert(kChunkBytes % 1024 == 0, "swizzle atoms must stay 1 KiB aligned");
+    static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+    static_assert(kSmemBytes > 114 * 1024, "one CTA per SM: each CTA owns all 512 TMEM columns");
+};
+
+struct Ctl {
+    volatile int32_t* abort_flag;
+    int32_t* err;
+};
+
+// Bounded wait on an mbarrier phase.  False: timed out (flag raised) or another role aborted.
+__device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, const Ctl& c) {
+    if (ptx::mbar_try_wait(bar, parity)) return true;
+    const long long t0 = clock64();
+    for (uint32_t n = 1;; ++n) {
+        if (ptx::mbar_try_wait(bar, parity)) return true;
+        if ((n & 63) == 0) {
+            if (*c.abort_flag) return false;
+            if (clock64() - t0 > kWaitLimitCycles) {
+                *c.abort_flag = 1;
+                atomicCAS(c.err, 0, RR_ERR_TIMEOUT);
+                return false;
+            }
+        }
+    }
+}
+
+// Bounded wait used only while draining after an abort (ignores the abort flag).
+__device__ __forceinline__ void drain_bar(uint32_t bar, uint32_t parity) {
+    const long long t0 = clock64();
+    while (!ptx::mbar_try_wait(bar, parity)) {
+        if (clock64() - t0 > (1ll << 31)) break;
+    }
+}
+
+// Snake order: even waves left to right, odd waves right to left.
+__device__ __forceinline__ int unit_of(int wave, int cta, int grid) {
+    return wave * grid + ((wave & 1) ? (grid - 1 - cta) : cta);
+}
+
+template <int D, int NS>
+__global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_constant__ AttnArgs a) {
+    using C = Cfg<D, NS>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const uint32_t sb = ptx::smem_u32(smem);
+    auto bar = [&](int i) -> uint32_t { return sb + C::kOffBar + 8u * (uint32_t)i; };
+    volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(smem + C::kOffMisc + 4);
+    const Ctl ctl{abort_flag, a.err};
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        ptx::mbar_init(bar(C::kQFull), 1);
+        ptx::mbar_init(bar(C::kQEmpty), 1);
+        for (int s = 0; s < NS; ++s) {
+            ptx::mbar_init(bar(C::kKFull + s), 1);
+            ptx::mbar_init(bar(C::kKEmpty + s), 1);
+            ptx::mbar_init(bar(C::kVFull + s), 1);
+            ptx::mbar_init(bar(C::kVEmpty + s), 1);
+        }
+        for (int q = 0; q < kNQ; ++q) {
+            ptx::mbar_init(bar(C::kSFull + q), 1);
+            ptx::mbar_init(bar(C::kPFull + q), kBM);
+            ptx::mbar_init(bar(C::kOFinal + q), 1);
+        }
+        ptx::mbar_init(bar(C::kVTmp), 1);
+        ptx::mbar_init(bar(C::kDrain), 1);
+        *abort_flag = 0;
+        ptx::fence_mbar_init();
+    }
+    if (warp == kWarpMMA) {
+        ptx::tmem_alloc(sb + C::kOffMisc, 512);
+        ptx::tmem_relinquish();
+    }
+    if (warp == kWarpProducer && lane == 0) {
+        ptx::prefetch_tmap(&a.tm_q);
+        ptx::prefetch_tmap(&a.tm_k);
+        ptx::prefetch_tmap(&a.tm_v);
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + C::kOffMisc);
+    const int n_units = *a.n_units;
+    const int grid = gridDim.x, cta = blockIdx.x;
+    const int unit_tokens = kNQ * a.tq;
+
+    if (warp == kWarpProducer) {
+        // ------------------------------------------------------------ TMA producer
+        const int ppt = kBN / a.ps;  // pages per KV tile (<= 16)
+        uint32_t kv_count = 0, unit_i = 0, vtmp_phase = 0;
+        // copies in flight, for the abort drain: bit s of armed_* = stage s armed, bit s of par_* = its parity
+        int armed_q = -1, armed_vtmp = -1;
+        uint32_t armed_k = 0, armed_v = 0, par_k = 0, par_v = 0;
+        bool ok = true;
+        for (int w = 0; ok; ++w) {
+            const int ui = unit_of(w, cta, grid);
+            if (ui >= n_units) break;
+            const int4 U = a.units[ui];
+            const int b = U.x, g = U.y, u = U.z, n_kv = U.w;
+            const int P = a.prefix[b], S = a.suffix[b], cu_b = a.cu[b];
+            const int t0 = u * unit_tokens;
+            const int n_keys = P + min(S, t0 + unit_tokens);
+            const int agent_len = P + S;
+            // Q tiles of this unit
+            if (lane == 0) {
+                if (unit_i > 0) ok = wait_bar(bar(C::kQEmpty), (unit_i - 1) & 1, ctl);
+                if (ok) {
+                    ptx::mbar_arrive_expect_tx(bar(C::kQFull), kNQ * C::kQTileBytes);
+                    for (int q = 0; q < kNQ; ++q)
+                        for (int c = 0; c < C::kChunks; ++c)
+                            ptx::tma_load_3d(sb + C::kOffQ + q * C::kQTileBytes + c * C::kChunkBytes, &a.tm_q,
+                                             c * 64, g * a.G, cu_b + t0 + q * a.tq, bar(C::kQFull));
+                    armed_q = (int)(unit_i & 1);
+                }
+            }
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            if (!ok) break;
+            const int last_page_end = ((n_keys + a.ps - 1) / a.ps) * a.ps;
+            for (int j = 0; j < n_kv; ++j, ++kv_count) {
+                const int s = (int)(kv_count % NS);
+                const uint32_t use = kv_count / NS;
+                int row = a.oob_row;  // page past the agent's keys: zero fill
+                if (lane < ppt) {
+                    const int lp = j * ppt + lane;
+                    if (lp * a.ps < n_keys) {
+                        const int pid = a.page_table[(long long)b * a.max_pages + lp];
+                        if (pid >= 0 && (long long)pid < a.num_pages) row = pid * a.ps;
+                        else atomicCAS(a.err, 0, RR_ERR_OOB);
+                    }
+                }
+                // K tile
+                if (lane == 0) {
+                    if (use > 0) ok = wait_bar(bar(C::kKEmpty + s), (use - 1) & 1, ctl);
+                    if (ok) ptx::mbar_arrive_expect_tx(bar(C::kKFull + s), C::kKVTileBytes);
+                }
+                ok = __shfl_sync(0xffffffffu, ok, 0);
+                if (!ok) break;
+                armed_k |= 1u << s;
+                par_k = (par_k & ~(1u << s)) | ((use & 1u) << s);
+                if (lane < ppt)
+                    for (int c = 0; c < C::kChunks; ++c)
+                        ptx::tma_load_2d(sb + C::kOffK + s * C::kKVTileBytes + c * C::kChunkBytes + lane * a.ps * 128,
+                                         &a.tm_k, g * D + c * 64, row, bar(C::kKFull + s));
+                // V tile; if the agent's last page is only partly its own, land it on the
+                // side barrier, clear the foreign slots, then release it to the MMA warp.
+                const bool clear_tail = (j == n_kv - 1) && (last_page_end > agent_len);
+                const uint32_t vbar = clear_tail ? bar(C::kVTmp) : bar(C::kVFull + s);
+                if (lane == 0) {
+                    if (use > 0) ok = wait_bar(bar(C::kVEmpty + s), (use - 1) & 1, ctl);
+                    if (ok) ptx::mbar_arrive_expect_tx(vbar, C::kKVTileBytes);
+                }
+                ok = __shfl_sync(0xffffffffu, ok, 0);
+                if (!ok) break;
+                if (lane < ppt)
+                    for (int c = 0; c < C::kChunks; ++c)
+                        ptx::tma_load_2d(sb + C::kOffV + s * C::kKVTileBytes + c * C::kChunkBytes + lane * a.ps * 128,
+                                         &a.tm_v, g * D + c * 64, row, vbar);
+                if (clear_tail) {
+                    armed_vtmp = (int)vtmp_phase;
+                    if (lane == 0) ok = wait_bar(bar(C::kVTmp), vtmp_phase, ctl);
+                    ok = __shfl_sync(0xffffffffu, ok, 0);
+                    if (!ok) break;
+                    armed_vtmp = -1;
+                    vtmp_phase ^= 1;
+                    const int r0 = agent_len - j * kBN;  // 0 < r0 < kBN: first row past the agent
+                    uint8_t* vt = smem + C::kOffV + s * C::kKVTileBytes;
+                    for (int c = 0; c < C::kChunks; ++c) {
+                        uint4* base = reinterpret_cast<uint4*>(vt + c * C::kChunkBytes);
+                        for (int e = r0 * 8 + lane; e < kBN * 8; e += 32) base[e] = make_uint4(0u, 0u, 0u, 0u);
+                    }
+                    ptx::fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) ptx::mbar_arrive(bar(C::kVFull + s));
+                } else {
+                    armed_v |= 1u << s;
+                    par_v = (par_v & ~(1u << s)) | ((use & 1u) << s);
+                }
+            }
+            ++unit_i;
+        }
+        if (!ok && lane == 0) {  // abort: let every copy this warp started land before exit
+            if (armed_q >= 0) drain_bar(bar(C::kQFull), (uint32_t)armed_q);
+            if (armed_vtmp >= 0) drain_bar(bar(C::kVTmp), (uint32_t)armed_vtmp);
+            for (int s = 0; s < NS; ++s) {
+                if (armed_k >> s & 1u) drain_bar(bar(C::kKFull + s), par_k >> s & 1u);
+                if (armed_v >> s & 1u) drain_bar(bar(C::kVFull + s), par_v >> s & 1u);
+            }
+        }
+        __syncwarp();
+    } else if (warp == kWarpMMA) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc_qk = ptx::idesc_bf16_f32(kBM, kBN, false, false);
+            constexpr uint32_t idesc_pv = ptx::idesc_bf16_f32(kBM, D, false, true);
+            uint32_t kv_count = 0, unit_i = 0;
+            uint32_t p_phase = 0;  // bit q: parity of the next P_q phase
+            bool ok = true;
+            auto issue_qk = [&](int q, int s) {
+                const uint32_t d_tmem = tmem + (uint32_t)(q * 128);
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk) {
+                    const uint32_t a_addr =
+                        sb + C::kOffQ + q * C::kQTileBytes + (kk >> 2) * C::kChunkBytes + (kk & 3) * 32;
+                    const uint32_t b_addr =
+                        sb + C::kOffK + s * C::kKVTileBytes + (kk >> 2) * C::kChunkBytes + (kk & 3) * 32;
+                    ptx::mma_ss(d_tmem, ptx::sdesc_sw128(a_addr, 16, 1024), ptx::sdesc_sw128(b_addr, 16, 1024),
+                                idesc_qk, kk > 0 ? 1u : 0u);
+                }
+            };
+            auto issue_pv = [&](int q, int s, bool accumulate) {
+                const uint32_t d_tmem = tmem + 256u + (uint32_t)(q * D);
+#pragma unroll
+                for (int kk = 0; kk < kBN / 16; ++kk) {
+                    const uint32_t a_tmem = tmem + (uint32_t)(q * 128 + kk * 8);  // P: bf16 pairs over S_q
+                    const uint32_t b_addr = sb + C::kOffV + s * C::kKVTileBytes + kk * 16 * 128;
+                    ptx::mma_ts(d_tmem, a_tmem, ptx::sdesc_sw128(b_addr, C::kChunkBytes, 1024), idesc_pv,
+                                (accumulate || kk > 0) ? 1u : 0u);
+                }
+            };
+            for (int w = 0; ok; ++w) {
+                const int ui = unit_of(w, cta, grid);
+                if (ui >= n_units) break;
+                const int n_kv = a.units[ui].w;
+                if (!(ok = wait_bar(bar(C::kQFull), unit_i & 1, ctl))) break;
+                ptx::tc_fence_after();
+                {
+                    const int s = (int)(kv_count % NS);
+                    if (!(ok = wait_bar(bar(C::kKFull + s), (kv_count / NS) & 1, ctl))) break;
+                    ptx::tc_fence_after();
+                    issue_qk(0, s);
+                    ptx::mma_commit(bar(C::kSFull + 0));
+                    issue_qk(1, s);
+                    ptx::mma_commit(bar(C::kSFull + 1));
+                    ptx::mma_commit(bar(C::kKEmpty + s));
+                }
+                for (int j = 0; j < n_kv && ok; ++j) {
+                    const uint32_t cur = kv_count + j, nxt = cur + 1;
+                    const int s = (int)(cur % NS), s1 = (int)(nxt % NS);
+                    const bool more = j + 1 < n_kv;
+                    if (!(ok = wait_bar(bar(C::kVFull + s), (cur / NS) & 1, ctl))) break;
+                    ptx::tc_fence_after();
+#pragma unroll
+                    for (int q = 0; q < kNQ; ++q) {
+                        if (!(ok = wait_bar(bar(C::kPFull + q), (p_phase >> q) & 1u, ctl))) break;
+                        p_phase ^= 1u << q;
+                        ptx::tc_fence_after();
+                        issue_pv(q, s, j > 0);
+                        if (!more) ptx::mma_commit(bar(C::kOFinal + q));
+                        if (more) {
+                            if (q == 0) {
+                                if (!(ok = wait_bar(bar(C::kKFull + s1), (nxt / NS) & 1, ctl))) break;
+                                ptx::tc_fence_after();
+                            }
+                            issue_qk(q, s1);
+                            ptx::mma_commit(bar(C::kSFull + q));
+                            if (q == kNQ - 1) ptx::mma_commit(bar(C::kKEmpty + s1));
+                        }
+                    }
+                    if (!ok) break;
+                    ptx::mma_commit(bar(C::kVEmpty + s));
+                }
+                if (!ok) break;
+                ptx::mma_commit(bar(C::kQEmpty));
+                kv_count += n_kv;
+                ++unit_i;
+            }
+            if (!ok) {  // abort: wait for every MMA this thread issued
+                ptx::mma_commit(bar(C::kDrain));
+                drain_bar(bar(C::kDrain), 0);
+            }
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ softmax warpgroups
+        const int q = warp >> 2;              // Q tile of this warpgroup
+        const int r = threadIdx.x & (kBM - 1);  // row == TMEM lane
+        const uint32_t lane_bits = (uint32_t)((warp & 3) * 32) << 16;
+        const uint32_t t_s = tmem + lane_bits + (uint32_t)(q * 128);
+        const uint32_t t_o = tmem + lane_bits + 256u + (uint32_t)(q * D);
+        const float sl2 = a.scale_log2;
+        uint32_t s_phase = 0, o_phase = 0;
+        bool ok = true;
+        for (int w = 0; ok; ++w) {
+            const int ui = unit_of(w, cta, grid);
+            if (ui >= n_units) break;
+            const int4 U = a.units[ui];
+            const int b = U.x, g = U.y, u = U.z, n_kv = U.w;
+            const int P = a.prefix[b], S = a.suffix[b], cu_b = a.cu[b];
+            const int tq0 = u * unit_tokens + q * a.tq;  // first suffix token of this Q tile
+            const int tok = tq0 + r / a.G;
+            const int head = g * a.G + r % a.G;
+            const int agent_len = P + S;
+            const int row_limit = min(P + tok, agent_len - 1);     // last key this row may see
+            const int mask_from = (min(P + tq0, agent_len - 1) + 1) / kBN;  // earlier tiles: no masking
+            float m_run = -INFINITY, l_run = 0.f;
+            for (int j = 0; j < n_kv; ++j) {
+                if (!(ok = wait_bar(bar(C::kSFull + q), s_phase, ctl))) break;
+                s_phase ^= 1;
+                ptx::tc_fence_after();
+                uint32_t sr[kBN];
+#pragma unroll
+                for (int c = 0; c < kBN; c += 32) ptx::tmem_ld32(t_s + c, *reinterpret_cast<uint32_t(*)[32]>(&sr[c]));
+                ptx::tmem_wait_ld();
+                float sv[kBN];
+#pragma unroll
+                for (int c = 0; c < kBN; ++c) sv[c] = __uint_as_float(sr[c]);
+                if (j >= mask_from) {
+                    const int lim = row_limit - j * kBN;
+#pragma unroll
+                    for (int c = 0; c < kBN; ++c)
+                        if (c > lim) sv[c] = -INFINITY;
+                }
+                float mx0 = sv[0], mx1 = sv[1], mx2 = sv[2], mx3 = sv[3];
+#pragma unroll
+                for (int c = 4; c < kBN; c += 4) {
+                    mx0 = fmaxf(mx0, sv[c]);
+                    mx1 = fmaxf(mx1, sv[c + 1]);
+                    mx2 = fmaxf(mx2, sv[c + 2]);
+                    mx3 = fmaxf(mx3, sv[c + 3]);
+                }
+                const float mxs = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2;
+                bool grow = false;
+                float f = 1.0f;
+                if (j == 0) {
+                    m_run = mxs;
+                } else if (mxs > m_run + 8.0f) {
+                    grow = true;
+                    f = ptx::ex2_approx(m_run - mxs);
+                    l_run *= f;
+                    m_run = mxs;
+                }
+                const float neg = -m_run;
+                float l0 = 0.f, l1 = 0.f;
+                uint32_t pk[kBN / 2];
+#pragma unroll
+                for (int c = 0; c < kBN; c += 2) {
+                    const float p0 = ptx::ex2_approx(fmaf(sv[c], sl2, neg));
+                    const float p1 = ptx::ex2_approx(fmaf(sv[c + 1], sl2, neg));
+                    l0 += p0;
+                    l1 += p1;
+                    pk[c >> 1] = ptx::pack_bf16x2(p0, p1);
+                }
+                l_run += l0 + l1;
+                ptx::tmem_st32(t_s, *reinterpret_cast<uint32_t(*)[32]>(&pk[0]));
+                ptx::tmem_st32(t_s + 32, *reinterpret_cast<uint32_t(*)[32]>(&pk[32]));
+                // O_q holds PV of tiles < j (complete: S_q(j) was issued after PV_q(j-1)); bring it to the
+                // new max before PV_q(j) may start, i.e. before this thread signals P_q(j).
+                if (__any_sync(0xffffffffu, grow)) {  // warp-uniform: tcgen05.ld/st are .sync.aligned
+#pragma unroll
+                    for (int c = 0; c < D; c += 32) {
+                        uint32_t o[32];
+                        ptx::tmem_ld32(t_o + c, o);
+                        ptx::tmem_wait_ld();
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * f);
+                        ptx::tmem_st32(t_o + c, o);
+                    }
+                }
+                ptx::tmem_wait_st();
+                ptx::tc_fence_before();
+                ptx::mbar_arrive(bar(C::kPFull + q));
+            }
+            if (!ok) break;
+            if (!(ok = wait_bar(bar(C::kOFinal + q), o_phase, ctl))) break;
+            o_phase ^= 1;
+            ptx::tc_fence_after();
+            const float inv_l = 1.0f / l_run;
+            const bool valid = tok < S;
+            __nv_bfloat16* dst =
+                reinterpret_cast<__nv_bfloat16*>(a.out) + ((long long)(cu_b + tok) * a.Hq + head) * D;
+#pragma unroll
+            for (int c = 0; c < D; c += 32) {
+                uint32_t o[32];
+                ptx::tmem_ld32(t_o + c, o);
+                ptx::tmem_wait_ld();
+                uint32_t pk[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i)
+                    pk[i] = ptx::pack_bf16x2(__uint_as_float(o[2 * i]) * inv_l, __uint_as_float(o[2 * i + 1]) * inv_l);
+                if (valid) {
+                    uint4* d4 = reinterpret_cast<uint4*>(dst + c);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) d4[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+                }
+            }
+        }
+    }
+
+    ptx::tc_fence_before();
+    __syncthreads();
+    if (warp == kWarpMMA) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem, 512);
+    }
+}
+
+template <int D, int NS>
+cudaError_t launch_cfg(const AttnArgs& a, int grid, cudaStream_t st) {
+    using C = Cfg<D, NS>;
+    static bool attr_done[64] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    if (!attr_done[dev]) {
+        e = cudaFuncSetAttribute(extend_attn_kernel<D, NS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 C::kSmemBytes);
+        if (e != cudaSuccess) return e;
+        attr_done[dev] = true;
+    }
+    extend_attn_kernel<D, NS><<<grid, kThreads, C::kSmemBytes, st>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+size_t extend_attention_smem_bytes(int head_dim) {
+    if (head_dim == 128) return Cfg<128, 2>::kSmemBytes;
+    if (head_dim == 64) return Cfg<64, 4>::kSmemBytes;
+    return 0;
+}
+
+cudaError_t launch_extend_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st) {
+    if (head_dim == 128) return launch_cfg<128, 2>(a, grid, st);
+    if (head_dim == 64) return launch_cfg<64, 4>(a, grid, st);
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace rr

@@ -1,0 +1,80 @@
+// kv_append.cu -- write the uncached suffix's K/V rows into the paged pool.
+//
+// Sec. 2: the prefill materialises the KV tensors of the tokens it processes;
+// the serving engine keeps them in a shared pool so the agent's next turn can
+// reuse them.  Suffix token j of agent b (row cu_b + j of k_new / v_new) goes
+// to position P_b + j: page page_table[b][pos / ps], slot pos % ps.
+//
+// One warp moves one token: the token's K row (all KV heads, Hkv*D bf16 =
+// 2 KiB at Hkv=8, D=128) is contiguous in k_new and contiguous in the pool
+// slot, so each lane issues 16-byte loads and stores that coalesce into whole
+// 512-byte warp transactions on both sides.  Pure HBM copy: 4*T*Hkv*D*2 bytes
+// of traffic, bound by HBM bandwidth.  The suffix rows are read once
+// (streaming loads); the pool writes keep the default policy because the
+// attention kernel reads those pages right after.
+#include "rr_internal.h"
+
+namespace rr {
+
+namespace {
+
+__device__ __forceinline__ int last_le(const int32_t* off, int n, long long x) {
+    int lo = 0, hi = n - 1;
+    while (lo < hi) {
+        int mid = (lo + hi + 1) >> 1;
+        if ((long long)off[mid] <= x) lo = mid; else hi = mid - 1;
+    }
+    return lo;
+}
+
+constexpr int kAppendThreads = 256;
+
+__global__ void __launch_bounds__(kAppendThreads) kv_append_kernel(const AppendArgs a) {
+    if (*a.lens_ok == 0) return;
+    const int lane = threadIdx.x & 31;
+    const long long warps = (long long)gridDim.x * (kAppendThreads / 32);
+    const uint4* __restrict__ kn = a.k_new;
+    const uint4* __restrict__ vn = a.v_new;
+    uint4* __restrict__ kp = a.k_pool;
+    uint4* __restrict__ vp = a.v_pool;
+    for (long long t = (long long)blockIdx.x * (kAppendThreads / 32) + (threadIdx.x >> 5); t < a.T; t += warps) {
+        const int b = last_le(a.cu, a.B, t);
+        const long long pos = (long long)a.prefix[b] + (t - a.cu[b]);
+        const int page = a.page_table[(long long)b * a.max_pages + pos / a.ps];
+        if (page < 0 || (long long)page >= a.num_pages) {
+            if (lane == 0) atomicCAS(a.err, 0, RR_ERR_OOB);
+            continue;
+        }
+        const long long src = t * a.row16;
+        const long long dst = ((long long)page * a.ps + pos % a.ps) * a.row16;
+        int e = lane;
+        for (; e + 96 < a.row16; e += 128) {  // four vectors of K and four of V in flight per lane
+            uint4 k0 = __ldcs(kn + src + e), k1 = __ldcs(kn + src + e + 32);
+            uint4 k2 = __ldcs(kn + src + e + 64), k3 = __ldcs(kn + src + e + 96);
+            uint4 v0 = __ldcs(vn + src + e), v1 = __ldcs(vn + src + e + 32);
+            uint4 v2 = __ldcs(vn + src + e + 64), v3 = __ldcs(vn + src + e + 96);
+            kp[dst + e] = k0; kp[dst + e + 32] = k1; kp[dst + e + 64] = k2; kp[dst + e + 96] = k3;
+            vp[dst + e] = v0; vp[dst + e + 32] = v1; vp[dst + e + 64] = v2; vp[dst + e + 96] = v3;
+        }
+        for (; e < a.row16; e += 32) {
+            uint4 k0 = __ldcs(kn + src + e);
+            uint4 v0 = __ldcs(vn + src + e);
+            kp[dst + e] = k0;
+            vp[dst + e] = v0;
+        }
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_kv_append(const AppendArgs& a, int sm_count, cudaStream_t st) {
+    const long long warps_needed = a.T;
+    long long blocks = (warps_needed + (kAppendThreads / 32) - 1) / (kAppendThreads / 32);
+    const long long cap = (long long)sm_count * 8;  // 8 resident blocks of 256 threads per SM
+    if (blocks > cap) blocks = cap;
+    if (blocks < 1) blocks = 1;
+    kv_append_kernel<<<(unsigned)blocks, kAppendThreads, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace rr

@@ -1,0 +1,389 @@
+// rr_api.cu -- the C ABI of librr.so (include/rr.h): argument validation,
+// the per-device workspace, TMA tensor-map encoding and kernel launches.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include <cudaTypedefs.h>
+
+#include "rr_internal.h"
+
+namespace {
+
+thread_local char g_msg[512] = "";
+
+int fail(int code, const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_msg, sizeof g_msg, fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+int cuda_fail(cudaError_t e, const char* what) {
+    return fail(RR_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+constexpr int kMaxDevices = 64;
+
+struct Device {
+    std::mutex mu;
+    bool init = false;
+    int sm_count = 0;
+    int32_t* err = nullptr;  // device error word (never moves once allocated)
+    void* ws = nullptr;      // schedule workspace, grown on demand
+    size_t ws_bytes = 0;
+};
+
+Device g_dev[kMaxDevices];
+std::mutex g_encode_mu;
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// Workspace layout: [n_units, lens_ok][cu: B+1][unit_off: B+1][units: max_units x int4]
+struct Layout {
+    size_t off_cu, off_unit_off, off_units, total;
+};
+
+Layout layout_for(int64_t B, int64_t max_units) {
+    Layout L;
+    L.off_cu = 256;
+    L.off_unit_off = L.off_cu + align256((size_t)(B + 1) * 4);
+    L.off_units = L.off_unit_off + align256((size_t)(B + 1) * 4);
+    L.total = L.off_units + align256((size_t)max_units * 16);
+    return L;
+}
+
+int current_device(Device** out, int* dev_out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= kMaxDevices) return fail(RR_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
+    Device& d = g_dev[dev];
+    std::lock_guard<std::mutex> lk(d.mu);
+    if (!d.init) {
+        e = cudaDeviceGetAttribute(&d.sm_count, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+        e = cudaMalloc(&d.err, 256);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaMalloc(error word)");
+        e = cudaMemset(d.err, 0, 256);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaMemset(error word)");
+        d.init = true;
+    }
+    *out = &d;
+    if (dev_out) *dev_out = dev;
+    return RR_OK;
+}
+
+// Make sure the workspace holds `bytes`.  Growing frees the old buffer, which
+// synchronises the device (so no kernel can still be using it).
+int ensure_ws(Device& d, size_t bytes) {
+    std::lock_guard<std::mutex> lk(d.mu);
+    if (d.ws_bytes >= bytes) return RR_OK;
+    if (d.ws) {
+        cudaError_t e = cudaFree(d.ws);
+        d.ws = nullptr;
+        d.ws_bytes = 0;
+        if (e != cudaSuccess) return cuda_fail(e, "cudaFree(workspace)");
+    }
+    size_t want = bytes + bytes / 4;
+    cudaError_t e = cudaMalloc(&d.ws, want);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMalloc(workspace)");
+    d.ws_bytes = want;
+    return RR_OK;
+}
+
+int get_encoder() {
+    std::lock_guard<std::mutex> lk(g_encode_mu);
+    if (g_encode) return RR_OK;
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn)
+        return fail(RR_ERR_CUDA, "cuTensorMapEncodeTiled entry point unavailable");
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    return RR_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+bool aligned4(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 3) == 0; }
+
+int check_dims(const rr_dims* d, bool attention) {
+    if (!d) return fail(RR_ERR_INVALID_ARG, "dims is null");
+    if (d->batch < 0 || d->total_tokens < 0 || d->num_pages < 0 || d->max_pages < 0)
+        return fail(RR_ERR_INVALID_ARG, "negative size in dims");
+    if (d->num_kv_heads <= 0 || d->num_q_heads <= 0 || d->num_q_heads % d->num_kv_heads)
+        return fail(RR_ERR_INVALID_ARG, "num_q_heads (%d) must be a positive multiple of num_kv_heads (%d)",
+                    d->num_q_heads, d->num_kv_heads);
+    if (d->head_dim != 64 && d->head_dim != 128)
+        return fail(RR_ERR_UNSUPPORTED, "head_dim %d unsupported (64 or 128)", d->head_dim);
+    const int ps = d->page_size;
+    if (ps != 8 && ps != 16 && ps != 32 && ps != 64 && ps != 128)
+        return fail(RR_ERR_UNSUPPORTED, "page_size %d unsupported (8, 16, 32, 64 or 128)", ps);
+    if (attention) {
+        const int G = d->num_q_heads / d->num_kv_heads;
+        if (G != 1 && G != 2 && G != 4 && G != 8 && G != 16)
+            return fail(RR_ERR_UNSUPPORTED, "GQA group %d unsupported (1, 2, 4, 8 or 16)", G);
+    }
+    if (d->total_tokens >= (1ll << 31)) return fail(RR_ERR_UNSUPPORTED, "total_tokens must be < 2^31");
+    if (d->num_pages * (int64_t)ps >= (1ll << 31) - ps)
+        return fail(RR_ERR_UNSUPPORTED, "num_pages * page_size must be < 2^31");
+    if (d->batch > 0 && d->max_pages == 0) return fail(RR_ERR_INVALID_ARG, "max_pages is 0");
+    return RR_OK;
+}
+
+int encode_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t row_stride_bytes,
+              uint32_t box_inner, uint32_t box_rows) {
+    cuuint64_t dims[2] = {inner, rows};
+    cuuint64_t strides[1] = {row_stride_bytes};
+    cuuint32_t box[2] = {box_inner, box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(RR_ERR_CUDA, "cuTensorMapEncodeTiled (2-D) failed: %d", (int)r);
+    return RR_OK;
+}
+
+int encode_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint64_t s1, uint64_t s2,
+              uint32_t b0, uint32_t b1, uint32_t b2) {
+    cuuint64_t dims[3] = {d0, d1, d2};
+    cuuint64_t strides[2] = {s1, s2};
+    cuuint32_t box[3] = {b0, b1, b2};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(RR_ERR_CUDA, "cuTensorMapEncodeTiled (3-D) failed: %d", (int)r);
+    return RR_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* rr_version(void) { return "rr-extend 0.1 (sm_103a)"; }
+
+const char* rr_last_error(void) { return g_msg; }
+
+int rr_kv_append(const void* k_new, const void* v_new, void* k_pool, void* v_pool, const int32_t* page_table,
+                 const int32_t* prefix_lens, const int32_t* suffix_lens, const rr_dims* dims, cudaStream_t stream) {
+    g_msg[0] = 0;
+    int rc = check_dims(dims, false);
+    if (rc) return rc;
+    if (dims->total_tokens == 0 && dims->batch == 0) return RR_OK;
+    if (!page_table || !prefix_lens || !suffix_lens) return fail(RR_ERR_INVALID_ARG, "null lens or page table");
+    if (dims->total_tokens > 0 && (!k_new || !v_new || !k_pool || !v_pool))
+        return fail(RR_ERR_INVALID_ARG, "null K/V pointer");
+    if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(k_pool) || !aligned16(v_pool))
+        return fail(RR_ERR_INVALID_ARG, "K/V pointers must be 16-byte aligned");
+    if (!aligned4(page_table) || !aligned4(prefix_lens) || !aligned4(suffix_lens))
+        return fail(RR_ERR_INVALID_ARG, "int32 arrays must be 4-byte aligned");
+    Device* d = nullptr;
+    if ((rc = current_device(&d, nullptr))) return rc;
+    const Layout L = layout_for(dims->batch, 0);
+    if ((rc = ensure_ws(*d, L.total))) return rc;
+    uint8_t* ws = static_cast<uint8_t*>(d->ws);
+
+    rr::SchedArgs s{};
+    s.prefix = prefix_lens;
+    s.suffix = suffix_lens;
+    s.B = dims->batch;
+    s.Hkv = dims->num_kv_heads;
+    s.unit_tokens = 1;
+    s.T = dims->total_tokens;
+    s.max_pages = dims->max_pages;
+    s.ps = dims->page_size;
+    s.max_units = 0;
+    s.build_units = 0;
+    s.cu = reinterpret_cast<int32_t*>(ws + L.off_cu);
+    s.unit_off = reinterpret_cast<int32_t*>(ws + L.off_unit_off);
+    s.units = nullptr;
+    s.n_units = reinterpret_cast<int32_t*>(ws);
+    s.lens_ok = reinterpret_cast<int32_t*>(ws) + 1;
+    s.err = d->err;
+    cudaError_t e = rr::launch_sched(s, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "schedule kernel launch");
+    if (dims->total_tokens == 0) return RR_OK;
+
+    rr::AppendArgs a{};
+    a.k_new = static_cast<const uint4*>(k_new);
+    a.v_new = static_cast<const uint4*>(v_new);
+    a.k_pool = static_cast<uint4*>(k_pool);
+    a.v_pool = static_cast<uint4*>(v_pool);
+    a.page_table = page_table;
+    a.prefix = prefix_lens;
+    a.cu = s.cu;
+    a.lens_ok = s.lens_ok;
+    a.err = d->err;
+    a.T = dims->total_tokens;
+    a.num_pages = dims->num_pages;
+    a.B = dims->batch;
+    a.max_pages = dims->max_pages;
+    a.ps = dims->page_size;
+    a.row16 = dims->num_kv_heads * dims->head_dim * 2 / 16;
+    e = rr::launch_kv_append(a, d->sm_count, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "kv_append kernel launch");
+    return RR_OK;
+}
+
+int rr_extend_attention(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
+                        const int32_t* prefix_lens, const int32_t* suffix_lens, void* out, const rr_dims* dims,
+                        float softmax_scale, cudaStream_t stream) {
+    g_msg[0] = 0;
+    int rc = check_dims(dims, true);
+    if (rc) return rc;
+    if (dims->total_tokens == 0 && dims->batch == 0) return RR_OK;
+    if (!page_table || !prefix_lens || !suffix_lens) return fail(RR_ERR_INVALID_ARG, "null lens or page table");
+    if (dims->total_tokens > 0 && (!q || !k_pool || !v_pool || !out))
+        return fail(RR_ERR_INVALID_ARG, "null q/pool/out pointer");
+    if (!aligned16(q) || !aligned16(k_pool) || !aligned16(v_pool) || !aligned16(out))
+        return fail(RR_ERR_INVALID_ARG, "q, pools and out must be 16-byte aligned");
+    if (!aligned4(page_table) || !aligned4(prefix_lens) || !aligned4(suffix_lens))
+        return fail(RR_ERR_INVALID_ARG, "int32 arrays must be 4-byte aligned");
+    if (dims->total_tokens > 0 && dims->num_pages == 0) return fail(RR_ERR_INVALID_ARG, "empty pool");
+    const int Hq = dims->num_q_heads, Hkv = dims->num_kv_heads, D = dims->head_dim, ps = dims->page_size;
+    const int G = Hq / Hkv;
+    const int tq = rr::kBM / G;
+    const int unit_tokens = rr::kNQ * tq;
+    const int64_t T = dims->total_tokens, B = dims->batch;
+    const int64_t max_units = (int64_t)Hkv * (T / unit_tokens + B + 1);
+    if (max_units >= (1ll << 31)) return fail(RR_ERR_UNSUPPORTED, "too many work units");
+
+    Device* d = nullptr;
+    if ((rc = current_device(&d, nullptr))) return rc;
+    if ((rc = get_encoder())) return rc;
+    const Layout L = layout_for(B, max_units);
+    if ((rc = ensure_ws(*d, L.total))) return rc;
+    uint8_t* ws = static_cast<uint8_t*>(d->ws);
+
+    rr::SchedArgs s{};
+    s.prefix = prefix_lens;
+    s.suffix = suffix_lens;
+    s.B = (int32_t)B;
+    s.Hkv = Hkv;
+    s.unit_tokens = unit_tokens;
+    s.T = T;
+    s.max_pages = dims->max_pages;
+    s.ps = ps;
+    s.max_units = max_units;
+    s.build_units = 1;
+    s.cu = reinterpret_cast<int32_t*>(ws + L.off_cu);
+    s.unit_off = reinterpret_cast<int32_t*>(ws + L.off_unit_off);
+    s.units = reinterpret_cast<int4*>(ws + L.off_units);
+    s.n_units = reinterpret_cast<int32_t*>(ws);
+    s.lens_ok = reinterpret_cast<int32_t*>(ws) + 1;
+    s.err = d->err;
+    cudaError_t e = rr::launch_sched(s, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "schedule kernel launch");
+    if (T == 0) return RR_OK;
+
+    rr::AttnArgs a;
+    memset(&a, 0, sizeof a);
+    if ((rc = encode_3d(&a.tm_q, q, (uint64_t)D, (uint64_t)Hq, (uint64_t)T, (uint64_t)D * 2, (uint64_t)Hq * D * 2, 64,
+                        (uint32_t)G, (uint32_t)tq)))
+        return rc;
+    const uint64_t rows = (uint64_t)dims->num_pages * (uint64_t)ps;
+    if ((rc = encode_2d(&a.tm_k, k_pool, (uint64_t)Hkv * D, rows, (uint64_t)Hkv * D * 2, 64, (uint32_t)ps))) return rc;
+    if ((rc = encode_2d(&a.tm_v, v_pool, (uint64_t)Hkv * D, rows, (uint64_t)Hkv * D * 2, 64, (uint32_t)ps))) return rc;
+    a.page_table = page_table;
+    a.prefix = prefix_lens;
+    a.suffix = suffix_lens;
+    a.cu = s.cu;
+    a.units = s.units;
+    a.n_units = s.n_units;
+    a.err = d->err;
+    a.out = out;
+    a.num_pages = dims->num_pages;
+    a.Hq = Hq;
+    a.G = G;
+    a.ps = ps;
+    a.max_pages = dims->max_pages;
+    a.tq = tq;
+    a.oob_row = (int32_t)rows;
+    const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)D);
+    a.scale_log2 = scale * 1.4426950408889634f;
+    const int64_t grid = std::min<int64_t>((int64_t)d->sm_count, max_units);
+    e = rr::launch_extend_attention(a, D, (int)std::max<int64_t>(grid, 1), stream);
+    if (e != cudaSuccess) return cuda_fail(e, "extend attention kernel launch");
+    return RR_OK;
+}
+
+int rr_validate_page_table(const int32_t* page_table, const int32_t* prefix_lens, const int32_t* suffix_lens,
+                           const rr_dims* dims) {
+    g_msg[0] = 0;
+    if (!dims) return fail(RR_ERR_INVALID_ARG, "dims is null");
+    if (dims->batch > 0 && (!page_table || !prefix_lens || !suffix_lens))
+        return fail(RR_ERR_INVALID_ARG, "null host array");
+    const int64_t ps = dims->page_size, np = dims->num_pages;
+    if (ps <= 0 || np < 0 || dims->max_pages < 0) return fail(RR_ERR_INVALID_ARG, "bad dims");
+    int64_t T = 0;
+    // owner[p]: -1 unused, else (agent << 1) | (page holds suffix positions)
+    std::vector<int64_t> owner((size_t)np, -1);
+    std::vector<uint8_t> shared_read((size_t)np, 0);
+    for (int32_t b = 0; b < dims->batch; ++b) {
+        const int64_t P = prefix_lens[b], S = suffix_lens[b];
+        if (P < 0 || S < 0 || P + S > (int64_t)dims->max_pages * ps)
+            return fail(RR_ERR_LENS, "agent %d: bad lengths (prefix %lld, suffix %lld)", b, (long long)P,
+                        (long long)S);
+        T += S;
+        const int64_t n = (P + S + ps - 1) / ps;
+        for (int64_t i = 0; i < n; ++i) {
+            const int64_t p = page_table[(int64_t)b * dims->max_pages + i];
+            if (p < 0 || p >= np) return fail(RR_ERR_OOB, "agent %d: page %lld of logical page %lld outside the pool",
+                                              b, (long long)p, (long long)i);
+            const bool writes = (i + 1) * ps > P && S > 0;  // holds at least one suffix position
+            if (writes) {
+                if (owner[(size_t)p] != -1 || shared_read[(size_t)p])
+                    return fail(RR_ERR_OVERLAP, "agent %d: suffix page %lld is also used elsewhere", b, (long long)p);
+                owner[(size_t)p] = ((int64_t)b << 1) | 1;
+            } else {
+                if (owner[(size_t)p] != -1 && (owner[(size_t)p] & 1))
+                    return fail(RR_ERR_OVERLAP, "agent %d: prefix page %lld is another agent's suffix page", b,
+                                (long long)p);
+                shared_read[(size_t)p] = 1;
+            }
+        }
+    }
+    if (T != dims->total_tokens)
+        return fail(RR_ERR_LENS, "sum of suffix lengths %lld != total_tokens %lld", (long long)T,
+                    (long long)dims->total_tokens);
+    return RR_OK;
+}
+
+int rr_get_device_error(cudaStream_t stream) {
+    Device* d = nullptr;
+    int rc = current_device(&d, nullptr);
+    if (rc) return rc;
+    cudaError_t e = cudaStreamSynchronize(stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    int32_t v = 0;
+    e = cudaMemcpy(&v, d->err, sizeof v, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy(error word)");
+    e = cudaMemset(d->err, 0, sizeof v);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemset(error word)");
+    return v;
+}
+
+void rr_shutdown(void) {
+    for (int i = 0; i < kMaxDevices; ++i) {
+        Device& d = g_dev[i];
+        std::lock_guard<std::mutex> lk(d.mu);
+        if (!d.init) continue;
+        int prev = 0;
+        cudaGetDevice(&prev);
+        cudaSetDevice(i);
+        if (d.ws) cudaFree(d.ws);
+        if (d.err) cudaFree(d.err);
+        d.ws = nullptr;
+        d.err = nullptr;
+        d.ws_bytes = 0;
+        d.init = false;
+        cudaSetDevice(prev);
+    }
+}
+
+}  // extern "C"

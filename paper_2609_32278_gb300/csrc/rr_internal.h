@@ -1,0 +1,77 @@
+// rr_internal.h -- declarations shared by the CUDA translation units of librr.so
+// (not part of the public ABI; the public ABI is include/rr.h).
+#pragma once
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "rr.h"
+
+namespace rr {
+
+// Tiling of the extend-attention kernel.
+constexpr int kBM = 128;          // packed (token, head) rows per Q tile = TMEM lanes
+constexpr int kBN = 128;          // keys per KV tile
+constexpr int kNQ = 2;            // Q tiles per work unit (two softmax warpgroups ping-pong)
+constexpr int kCostBuckets = 4096;  // schedule: counting sort on the number of KV tiles
+
+// Device-side bookkeeping of one call (all pointers into the per-device workspace).
+struct SchedArgs {
+    const int32_t* prefix;
+    const int32_t* suffix;
+    int32_t B, Hkv;
+    int32_t unit_tokens;   // suffix tokens covered by one work unit (kNQ * kBM / G)
+    int64_t T;
+    int32_t max_pages, ps;
+    int64_t max_units;
+    int32_t build_units;   // 0: lengths prefix sums only (append)
+    int32_t* cu;           // [B+1] exclusive prefix sum of suffix lens
+    int32_t* unit_off;     // [B+1] first work unit of each agent
+    int4* units;           // [max_units] (agent, kv head, unit index, KV tiles), most expensive first
+    int32_t* n_units;
+    int32_t* lens_ok;
+    int32_t* err;
+};
+
+struct AppendArgs {
+    const uint4* k_new;
+    const uint4* v_new;
+    uint4* k_pool;
+    uint4* v_pool;
+    const int32_t* page_table;
+    const int32_t* prefix;
+    const int32_t* cu;
+    const int32_t* lens_ok;
+    int32_t* err;
+    int64_t T;
+    int64_t num_pages;
+    int32_t B, max_pages, ps;
+    int32_t row16;         // 16-byte vectors per token row (Hkv * D * 2 / 16)
+};
+
+struct AttnArgs {
+    CUtensorMap tm_q;      // q   [T][Hq][D]        box {64, G, 128/G}, 128B swizzle
+    CUtensorMap tm_k;      // k_pool [pages*ps][Hkv*D] box {64, ps},   128B swizzle
+    CUtensorMap tm_v;      // v_pool, same
+    const int32_t* page_table;
+    const int32_t* prefix;
+    const int32_t* suffix;
+    const int32_t* cu;
+    const int4* units;
+    const int32_t* n_units;
+    int32_t* err;
+    void* out;             // [T][Hq][D] bf16
+    int64_t num_pages;
+    int32_t Hq, G, ps, max_pages;
+    int32_t tq;            // tokens per Q tile = 128 / G
+    int32_t oob_row;       // first row past the pool (TMA fills it with zeros)
+    float scale_log2;      // softmax scale * log2(e)
+};
+
+cudaError_t launch_sched(const SchedArgs& a, cudaStream_t st);
+cudaError_t launch_kv_append(const AppendArgs& a, int sm_count, cudaStream_t st);
+// Returns cudaErrorInvalidValue for an unsupported head dim.
+cudaError_t launch_extend_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st);
+size_t extend_attention_smem_bytes(int head_dim);
+
+}  // namespace rr

@@ -1,0 +1,92 @@
+"""Shared helpers of the GPU parity tests: tolerance check, row sampling, oracle on sampled rows."""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+import oracle
+import synth
+
+# Attention parity bar (bf16 inputs, fp32 accumulation): fp64 oracle vs the bf16 output.
+MAX_ABS = 1e-2
+MEAN_ABS = 1e-3
+
+
+def bf16_bits(t) -> np.ndarray:
+    import torch
+    return t.detach().contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+def to_f64(t) -> np.ndarray:
+    return synth.bf16_to_f64(bf16_bits(t))
+
+
+def check_close(got: np.ndarray, ref: np.ndarray, what: str = "") -> dict:
+    err = np.abs(got - ref)
+    stats = dict(n=int(err.size), max=float(err.max()) if err.size else 0.0,
+                 mean=float(err.mean()) if err.size else 0.0,
+                 p999=float(np.quantile(err, 0.999)) if err.size else 0.0)
+    assert np.isfinite(got).all(), f"{what}: non-finite outputs"
+    assert stats["max"] <= MAX_ABS and stats["mean"] <= MEAN_ABS, f"{what}: {stats}"
+    return stats
+
+
+def sample_rows(wl: synth.Workload, flop_budget: float = 4e11, seed: int = 0):
+    """Suffix rows (agent, row) to check on a full-size config, within an fp64 flop budget.
+
+    Every agent's first and last row; one window of consecutive rows of the
+    agent with the longest prefix (covers every row position of two Q tiles);
+    then seeded random rows while the budget lasts.
+    """
+    rng = np.random.default_rng(seed)
+    cost = lambda b: 4.0 * wl.D * wl.Hq * (int(wl.prefix_lens[b]) + int(wl.suffix_lens[b]))
+    picked = {b: set() for b in range(wl.B)}
+    spent = 0.0
+    for b in range(wl.B):
+        S = int(wl.suffix_lens[b])
+        if S == 0:
+            continue
+        for i in {0, S - 1}:
+            picked[b].add(i)
+            spent += cost(b)
+    live = [b for b in range(wl.B) if wl.suffix_lens[b] > 0]
+    if live:
+        bw = max(live, key=lambda b: int(wl.prefix_lens[b]))
+        window = min(int(wl.suffix_lens[bw]), 2 * 128 // wl.G + 5)
+        for i in range(window):
+            if i not in picked[bw]:
+                picked[bw].add(i)
+                spent += cost(bw)
+    tries = 0
+    while spent < flop_budget and live and tries < 100000:
+        tries += 1
+        b = int(rng.choice(live))
+        i = int(rng.integers(0, int(wl.suffix_lens[b])))
+        if i in picked[b]:
+            continue
+        picked[b].add(i)
+        spent += cost(b)
+    return {b: np.array(sorted(v), dtype=np.int64) for b, v in picked.items() if v}
+
+
+def oracle_sampled(wl: synth.Workload, rows_by_agent, scale=None, nthreads=0):
+    """fp64 oracle on sampled rows from logically generated K/V (never from a pool).
+
+    Returns {agent: array [n_rows, Hq, D]} for the rows in rows_by_agent.
+    """
+    if scale is None:
+        scale = 1.0 / math.sqrt(wl.D)
+    out = {}
+    for b, rows in rows_by_agent.items():
+        P = int(wl.prefix_lens[b])
+        pos = P + rows
+        L = int(pos.max()) + 1
+        qr = synth.q_rows(wl, b, pos, nthreads)
+        res = np.zeros((len(rows), wl.Hq, wl.D))
+        for g in range(wl.Hkv):
+            K, V = synth.agent_kv(wl, b, L, g, nthreads)
+            res[:, g * wl.G:(g + 1) * wl.G] = oracle.attention_rows(qr[:, g * wl.G:(g + 1) * wl.G], pos, K, V,
+                                                                   scale, nthreads)
+        out[b] = res
+    return out

@@ -1,0 +1,193 @@
+"""Extend attention on the GPU vs the fp64 oracle, element by element, plus the invariants.
+
+Sizes here are small enough for the oracle to check every output element,
+while still spanning several KV tiles, several work units, ragged last Q tiles,
+mid-page prefixes and every supported GQA group and head dim.  Every pool slot
+that no agent owns holds a NaN, so reading one would poison the output.
+"""
+import math
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from parity import bf16_bits, check_close, to_f64
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def rr():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    import paper_2609_32278_gb300 as m
+    m.lib()
+    return m
+
+
+def run_gpu(rr, wl, g=None, scale=0.0):
+    if g is None:
+        g = synth.gpu_tensors(wl, "cuda")
+    rr.kv_append(g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                 g["suffix_lens"])
+    out = rr.extend_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                              g["suffix_lens"], softmax_scale=scale)
+    assert rr.device_error() == 0, rr.last_error()
+    return out, g
+
+
+def run_oracle(wl, scale=None, t=None):
+    t = t if t is not None else synth.cpu_tensors(wl)
+    kp, vp = oracle.kv_append(t["k_new"], t["v_new"], t["k_pool"], t["v_pool"], wl.page_table, wl.prefix_lens,
+                              wl.suffix_lens)
+    return oracle.extend_attention(t["q"], kp, vp, wl.page_table, wl.prefix_lens, wl.suffix_lens, scale=scale)
+
+
+CASES = [
+    # name, B, Hq, Hkv, D, prefix, suffix
+    ("d128_g4_basic", 2, 8, 2, 128, [256, 512], [64, 100]),
+    ("d128_g4_ragged_midpage", 3, 8, 2, 128, [37, 300, 0], [129, 70, 200]),
+    ("d128_g8", 2, 16, 2, 128, [700, 33], [90, 41]),
+    ("d128_g1", 2, 2, 2, 128, [150, 0], [300, 257]),
+    ("d128_g2", 2, 4, 2, 128, [1000, 64], [130, 5]),
+    ("d128_g16", 1, 16, 1, 128, [77], [40]),
+    ("d64_g4", 3, 8, 2, 64, [128, 999, 16], [33, 66, 130]),
+    ("d64_g1", 2, 2, 2, 64, [3, 250], [129, 1]),
+    ("suffix_one_token", 3, 8, 2, 128, [1023, 0, 5], [1, 1, 1]),
+    ("no_prefix", 2, 8, 2, 128, [0, 0], [255, 513]),
+    ("zero_suffix_agents", 4, 8, 2, 128, [64, 300, 50, 0], [0, 70, 0, 33]),
+    ("page_boundaries", 3, 8, 2, 128, [127, 128, 129], [1, 127, 128]),
+]
+
+
+@pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
+def test_attention_matches_oracle(rr, case):
+    name, B, Hq, Hkv, D, P, S = case
+    wl = synth.custom(name, B, Hq, Hkv, D, P, S, seed=3)
+    out, _ = run_gpu(rr, wl)
+    ref = run_oracle(wl, 1.0 / math.sqrt(D))
+    check_close(to_f64(out), ref, name)
+
+
+def test_c1_tiny_all_rows(rr):
+    wl = synth.config("c1_tiny")
+    out, _ = run_gpu(rr, wl)
+    ref = run_oracle(wl, 1.0 / math.sqrt(wl.D))
+    stats = check_close(to_f64(out), ref, "c1_tiny")
+    assert stats["n"] == wl.T * wl.Hq * wl.D
+
+
+def test_custom_scale(rr):
+    wl = synth.custom("scale", 2, 8, 2, 128, [200, 10], [60, 130], seed=5)
+    out, _ = run_gpu(rr, wl, scale=0.03)
+    check_close(to_f64(out), run_oracle(wl, 0.03), "scale")
+
+
+def test_page_permutation_is_bit_exact(rr):
+    # I2 on the GPU: a different physical placement gives identical output bits
+    a = synth.custom("pa", 3, 8, 2, 128, [300, 45, 512], [70, 200, 33], seed=8, num_pages=200)
+    b = synth.custom("pb", 3, 8, 2, 128, [300, 45, 512], [70, 200, 33], seed=8, num_pages=331)
+    assert not np.array_equal(a.page_table, b.page_table)
+    oa, _ = run_gpu(rr, a)
+    ob, _ = run_gpu(rr, b)
+    np.testing.assert_array_equal(bf16_bits(oa), bf16_bits(ob))
+
+
+def test_agent_order_permutation_permutes_rows(rr):
+    P, S = [300, 45, 512, 0], [70, 200, 33, 129]
+    a = synth.custom("oa", 4, 8, 2, 128, P, S, seed=8)
+    oa, _ = run_gpu(rr, a)
+    perm = [2, 0, 3, 1]
+    # same logical agents listed in another order (agent identity follows the generator's owner index)
+    g = synth.gpu_tensors(a, "cuda")
+    import torch
+    cu = a.cu
+    rows = np.concatenate([np.arange(cu[b], cu[b + 1]) for b in perm])
+    ridx = torch.from_numpy(rows).cuda()
+    g2 = dict(g)
+    for k in ("q", "k_new", "v_new"):
+        g2[k] = g[k][ridx].contiguous()
+    pidx = torch.tensor(perm).cuda()
+    for k in ("page_table", "prefix_lens", "suffix_lens"):
+        g2[k] = g[k][pidx].contiguous()
+    ob, _ = run_gpu(rr, a, g=g2)
+    np.testing.assert_array_equal(bf16_bits(ob), bf16_bits(oa)[rows])
+
+
+def test_unit_values_give_unit_output(rr):
+    import torch
+    wl = synth.custom("ones", 2, 8, 2, 128, [333, 64], [150, 70], seed=9)
+    g = synth.gpu_tensors(wl, "cuda")
+    g["v_new"].fill_(1.0)
+    for b in range(wl.B):
+        for lp in range(-(-int(wl.prefix_lens[b]) // wl.ps)):
+            g["v_pool"][int(wl.page_table[b, lp])] = 1.0
+    out, _ = run_gpu(rr, wl, g=g)
+    # o = sum_j bf16(p_j) / sum_j p_j: within one bf16 step of 1 (the weights are rounded to bf16 for the MMA)
+    np.testing.assert_allclose(to_f64(out), 1.0, rtol=0, atol=2 ** -8)
+    del torch
+
+
+def test_prefix_extend_matches_full_causal(rr):
+    # I1 on the GPU: extend(P, S) rows vs from-scratch causal attention over P + S, last S rows
+    P, S = [400, 129], [100, 200]
+    ext = synth.custom("ext", 2, 8, 2, 128, P, S, seed=21)
+    full = synth.custom("full", 2, 8, 2, 128, [0, 0], [p + s for p, s in zip(P, S)], seed=21)
+    oe, _ = run_gpu(rr, ext)
+    of, _ = run_gpu(rr, full)
+    fe, ff = to_f64(oe), to_f64(of)
+    for b in range(2):
+        a0, a1 = ext.cu[b], ext.cu[b + 1]
+        f1 = full.cu[b + 1]
+        d = np.abs(fe[a0:a1] - ff[f1 - S[b]:f1])
+        assert d.max() <= 2e-2 and d.mean() <= 1e-3
+
+
+def test_long_prefix_many_tiles(rr):
+    wl = synth.custom("long", 1, 8, 2, 128, [6000], [300], seed=12)
+    out, _ = run_gpu(rr, wl)
+    check_close(to_f64(out), run_oracle(wl, 1 / math.sqrt(128)), "long")
+
+
+def test_lens_mismatch_is_a_device_error(rr):
+    wl = synth.custom("lm", 2, 8, 2, 128, [64, 0], [10, 20], seed=2)
+    g = synth.gpu_tensors(wl, "cuda")
+    sl = g["suffix_lens"].clone()
+    sl[0] = 11
+    rr.extend_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"], sl)
+    assert rr.device_error() == rr.RR_ERR_LENS
+
+
+def test_bad_page_is_a_device_error(rr):
+    wl = synth.custom("bp", 2, 8, 2, 128, [64, 0], [10, 20], seed=2)
+    g = synth.gpu_tensors(wl, "cuda")
+    pt = g["page_table"].clone()
+    pt[0, 1] = -7
+    rr.extend_attention(g["q"], g["k_pool"], g["v_pool"], pt, g["prefix_lens"], g["suffix_lens"])
+    assert rr.device_error() == rr.RR_ERR_OOB
+
+
+def test_unsupported_shapes_are_rejected(rr):
+    import torch
+    q = torch.zeros((4, 3, 128), dtype=torch.bfloat16, device="cuda")
+    pool = torch.zeros((4, 16, 1, 128), dtype=torch.bfloat16, device="cuda")
+    pt = torch.zeros((1, 1), dtype=torch.int32, device="cuda")
+    lens = torch.tensor([4], dtype=torch.int32, device="cuda")
+    with pytest.raises(rr.RRError) as e:
+        rr.extend_attention(q, pool, pool, pt, lens * 0, lens)   # G = 3
+    assert e.value.code == rr.RR_ERR_UNSUPPORTED
+    q96 = torch.zeros((4, 2, 96), dtype=torch.bfloat16, device="cuda")
+    pool96 = torch.zeros((4, 16, 1, 96), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(rr.RRError) as e:
+        rr.extend_attention(q96, pool96, pool96, pt, lens * 0, lens)
+    assert e.value.code == rr.RR_ERR_UNSUPPORTED
+
+
+def test_gpu_generator_matches_cpu(rr):
+    wl = synth.custom("gen", 3, 8, 2, 128, [40, 0, 77], [9, 30, 1], seed=31, shared_len=32)
+    g = synth.gpu_tensors(wl, "cuda")
+    t = synth.cpu_tensors(wl)
+    for k in ("q", "k_new", "v_new", "k_pool", "v_pool"):
+        np.testing.assert_array_equal(bf16_bits(g[k]), t[k])
