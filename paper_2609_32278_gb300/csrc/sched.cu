@@ -76,7 +76,7 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     const long long tot_s = s_ws[31], tot_u = s_wu[31];
     long long off_s = (warp ? s_ws[warp - 1] : 0) + inc_s - sum_s;
     long long off_u = (warp ? s_wu[warp - 1] : 0) + inc_u - sum_u;
-    const bool ok = !s_bad && tot_s == a.T && tot_u <= a.max_units && tot_s < (1ll << 31);
+    const bool ok = !s_bad && tot_s == a.T && tot_s < (1ll << 31) && (!a.build_units || tot_u <= a.max_units);
     if (ok) {
         for (int b = b0; b < b1; ++b) {
             const long long S = a.suffix[b];
