@@ -32,25 +32,35 @@ def check_close(got: np.ndarray, ref: np.ndarray, what: str = "") -> dict:
     return stats
 
 
-def sample_rows(wl: synth.Workload, flop_budget: float = 4e11, seed: int = 0):
+def sample_rows(wl: synth.Workload, flop_budget: float = 4e11, seed: int = 0, max_agents: int = 12):
     """Suffix rows (agent, row) to check on a full-size config, within an fp64 flop budget.
 
-    Every agent's first and last row; one window of consecutive rows of the
-    agent with the longest prefix (covers every row position of two Q tiles);
-    then seeded random rows while the budget lasts.
+    Agents: all of them if there are at most `max_agents`, else the agents with
+    the longest prefix, the longest suffix and the shortest context plus seeded
+    random others (regenerating each sampled agent's K/V on the CPU is the
+    expensive part).  Rows: each sampled agent's first and last row; one window
+    of consecutive rows of the agent with the longest prefix (covers every row
+    position of two Q tiles); then seeded random rows while the budget lasts.
     """
     rng = np.random.default_rng(seed)
     cost = lambda b: 4.0 * wl.D * wl.Hq * (int(wl.prefix_lens[b]) + int(wl.suffix_lens[b]))
-    picked = {b: set() for b in range(wl.B)}
+    live_all = [b for b in range(wl.B) if wl.suffix_lens[b] > 0]
+    if len(live_all) > max_agents:
+        must = {max(live_all, key=lambda b: int(wl.prefix_lens[b])),
+                max(live_all, key=lambda b: int(wl.suffix_lens[b])),
+                min(live_all, key=lambda b: int(wl.prefix_lens[b]) + int(wl.suffix_lens[b]))}
+        rest = [b for b in live_all if b not in must]
+        extra = rng.choice(rest, size=max(0, max_agents - len(must)), replace=False)
+        live = sorted(must | set(int(x) for x in extra))
+    else:
+        live = live_all
+    picked = {b: set() for b in live}
     spent = 0.0
-    for b in range(wl.B):
+    for b in live:
         S = int(wl.suffix_lens[b])
-        if S == 0:
-            continue
         for i in {0, S - 1}:
             picked[b].add(i)
             spent += cost(b)
-    live = [b for b in range(wl.B) if wl.suffix_lens[b] > 0]
     if live:
         bw = max(live, key=lambda b: int(wl.prefix_lens[b]))
         window = min(int(wl.suffix_lens[bw]), 2 * 128 // wl.G + 5)
