@@ -112,6 +112,43 @@ int rr_extend_attention(const void* q, const void* k_pool, const void* v_pool, c
                         float softmax_scale, cudaStream_t stream);
 
 /*
+ * rr_extend_attention_noalloc -- rr_extend_attention for callers that cannot
+ * allocate device memory.  The paper has no counterpart; this is a deployment
+ * convenience of this library.
+ *
+ * Some callers must not allocate during a call: a serving engine whose device
+ * memory is entirely owned by its own pool allocator (the KV pool takes nearly
+ * all of HBM), or a latency-critical loop that cannot afford the implicit
+ * device-wide synchronisation of cudaMalloc/cudaFree.  This entry point
+ * computes exactly what rr_extend_attention computes (same kernels, same
+ * arguments and layouts), but keeps its schedule scratch in one fixed array
+ * of static device memory (about 1.06 MiB) that every GPU loading the library
+ * holds until the process exits.  It calls no cudaMalloc, cudaFree or other
+ * allocating routine.
+ *
+ * Limits: at most 4096 agents, and at most 65536 schedule work units, where
+ * the units needed are bounded by Hkv * (T / (256 / G) + B + 1).  Larger
+ * batches return RR_ERR_UNSUPPORTED without launching anything.
+ *
+ * device_error: optional device int32 (4-byte aligned) that receives a
+ * device-side error code (RR_ERR_LENS, RR_ERR_OOB, RR_ERR_TIMEOUT) if one
+ * occurs; the kernels only ever write a nonzero code into it when it is still
+ * zero, so the caller clears it.  With NULL, such errors are not reported.
+ *
+ * The first call on a device looks up the device address of the static array
+ * (cudaGetSymbolAddress) and the device's SM count; make that first call
+ * before any stream capture.  All calls on a device share the one array and
+ * it keeps the last call's contents (every field is rewritten by each call
+ * before it is read), so calls that overlap on the GPU -- on different
+ * streams, or from different threads without ordering -- race on it and must
+ * not be issued.
+ */
+int rr_extend_attention_noalloc(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
+                                const int32_t* prefix_lens, const int32_t* suffix_lens, void* out,
+                                const rr_dims* dims, float softmax_scale, int32_t* device_error,
+                                cudaStream_t stream);
+
+/*
  * rr_validate_page_table -- HOST-side check of a page table before use
  * (host arrays, not device).  Returns RR_OK, RR_ERR_LENS (bad lengths),
  * RR_ERR_OOB (a page an agent uses is outside [0, num_pages)) or

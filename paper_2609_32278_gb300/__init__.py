@@ -31,7 +31,7 @@ RR_ERR_OVERLAP = 7
 
 # Every symbol include/rr.h declares.
 EXPORTS = ("rr_kv_append", "rr_extend_attention", "rr_validate_page_table", "rr_get_device_error",
-           "rr_last_error", "rr_version", "rr_shutdown")
+           "rr_last_error", "rr_version", "rr_shutdown", "rr_extend_attention_noalloc")
 
 
 class RRError(RuntimeError):

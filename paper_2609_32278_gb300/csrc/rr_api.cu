@@ -387,3 +387,147 @@ void rr_shutdown(void) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// rr_extend_attention_noalloc: the same extend attention, with its schedule
+// scratch in a fixed static device array instead of the growable workspace.
+//
+// For callers that must not allocate device memory during a call: code that
+// runs inside a memory-budgeted serving loop or a custom allocator that owns
+// every device byte, or that cannot tolerate the implicit device
+// synchronisation of cudaMalloc/cudaFree.  The array below is part of the
+// library image: every GPU that loads librr.so holds it until process exit.
+namespace {
+
+constexpr int32_t kNoAllocMaxBatch = 4096;    // agents per call
+constexpr int64_t kNoAllocMaxUnits = 65536;   // schedule work units per call
+constexpr size_t kNoAllocOffCu = 256;         // [0] n_units, [1] lens_ok, [2] spare error word
+constexpr size_t kNoAllocOffUnitOff = kNoAllocOffCu + ((size_t)(kNoAllocMaxBatch + 1) * 4 + 255) / 256 * 256;
+constexpr size_t kNoAllocOffUnits = kNoAllocOffUnitOff + ((size_t)(kNoAllocMaxBatch + 1) * 4 + 255) / 256 * 256;
+constexpr size_t kNoAllocBytes = kNoAllocOffUnits + (size_t)kNoAllocMaxUnits * 16;  // ~1.06 MiB
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
+
+struct NoAllocDevice {
+    std::mutex mu;
+    bool ready = false;
+    void* scratch = nullptr;  // device address of g_noalloc_scratch on this device
+    int sm_count = 0;
+};
+NoAllocDevice g_noalloc[kMaxDevices];
+
+// One-time set-up per device, with that device current: the device address of
+// the static array (its host-side name is only a stand-in) and the SM count.
+int noalloc_setup(void** scratch, int* sm_count) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= kMaxDevices) return fail(RR_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
+    NoAllocDevice& d = g_noalloc[dev];
+    std::lock_guard<std::mutex> lk(d.mu);
+    if (!d.ready) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess || p == nullptr) return cuda_fail(e, "cudaGetSymbolAddress(static scratch)");
+        int sms = 0;
+        e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+        d.scratch = p;
+        d.sm_count = sms;
+        d.ready = true;
+    }
+    *scratch = d.scratch;
+    *sm_count = d.sm_count;
+    return RR_OK;
+}
+
+}  // namespace
+
+extern "C" int rr_extend_attention_noalloc(const void* q, const void* k_pool, const void* v_pool,
+                                           const int32_t* page_table, const int32_t* prefix_lens,
+                                           const int32_t* suffix_lens, void* out, const rr_dims* dims,
+                                           float softmax_scale, int32_t* device_error, cudaStream_t stream) {
+    g_msg[0] = 0;
+    int rc = check_dims(dims, true);
+    if (rc) return rc;
+    if (dims->total_tokens == 0 && dims->batch == 0) return RR_OK;
+    if (!page_table || !prefix_lens || !suffix_lens) return fail(RR_ERR_INVALID_ARG, "null lens or page table");
+    if (dims->total_tokens > 0 && (!q || !k_pool || !v_pool || !out))
+        return fail(RR_ERR_INVALID_ARG, "null q/pool/out pointer");
+    if (!aligned16(q) || !aligned16(k_pool) || !aligned16(v_pool) || !aligned16(out))
+        return fail(RR_ERR_INVALID_ARG, "q, pools and out must be 16-byte aligned");
+    if (!aligned4(page_table) || !aligned4(prefix_lens) || !aligned4(suffix_lens) || !aligned4(device_error))
+        return fail(RR_ERR_INVALID_ARG, "int32 arrays must be 4-byte aligned");
+    if (dims->total_tokens > 0 && dims->num_pages == 0) return fail(RR_ERR_INVALID_ARG, "empty pool");
+    const int Hq = dims->num_q_heads, Hkv = dims->num_kv_heads, D = dims->head_dim, ps = dims->page_size;
+    const int G = Hq / Hkv;
+    const int tq = rr::kBM / G;
+    const int unit_tokens = rr::kNQ * tq;
+    const int64_t T = dims->total_tokens, B = dims->batch;
+    const int64_t max_units = (int64_t)Hkv * (T / unit_tokens + B + 1);
+    if (B > kNoAllocMaxBatch)
+        return fail(RR_ERR_UNSUPPORTED, "batch %lld exceeds the static scratch limit of %d agents", (long long)B,
+                    kNoAllocMaxBatch);
+    if (max_units > kNoAllocMaxUnits)
+        return fail(RR_ERR_UNSUPPORTED,
+                    "batch needs up to %lld work units; the static scratch holds %lld (fewer suffix tokens per call)",
+                    (long long)max_units, (long long)kNoAllocMaxUnits);
+
+    void* scratch = nullptr;
+    int sm_count = 0;
+    if ((rc = noalloc_setup(&scratch, &sm_count))) return rc;
+    if ((rc = get_encoder())) return rc;
+    uint8_t* ws = static_cast<uint8_t*>(scratch);
+    int32_t* err = device_error ? device_error : reinterpret_cast<int32_t*>(ws) + 2;
+
+    rr::SchedArgs s{};
+    s.prefix = prefix_lens;
+    s.suffix = suffix_lens;
+    s.B = (int32_t)B;
+    s.Hkv = Hkv;
+    s.unit_tokens = unit_tokens;
+    s.T = T;
+    s.max_pages = dims->max_pages;
+    s.ps = ps;
+    s.max_units = max_units;
+    s.build_units = 1;
+    s.cu = reinterpret_cast<int32_t*>(ws + kNoAllocOffCu);
+    s.unit_off = reinterpret_cast<int32_t*>(ws + kNoAllocOffUnitOff);
+    s.units = reinterpret_cast<int4*>(ws + kNoAllocOffUnits);
+    s.n_units = reinterpret_cast<int32_t*>(ws);
+    s.lens_ok = reinterpret_cast<int32_t*>(ws) + 1;
+    s.err = err;
+    cudaError_t e = rr::launch_sched(s, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "schedule kernel launch");
+    if (T == 0) return RR_OK;
+
+    rr::AttnArgs a;
+    memset(&a, 0, sizeof a);
+    if ((rc = encode_3d(&a.tm_q, q, (uint64_t)D, (uint64_t)Hq, (uint64_t)T, (uint64_t)D * 2, (uint64_t)Hq * D * 2, 64,
+                        (uint32_t)G, (uint32_t)tq)))
+        return rc;
+    const uint64_t rows = (uint64_t)dims->num_pages * (uint64_t)ps;
+    if ((rc = encode_2d(&a.tm_k, k_pool, (uint64_t)Hkv * D, rows, (uint64_t)Hkv * D * 2, 64, (uint32_t)ps))) return rc;
+    if ((rc = encode_2d(&a.tm_v, v_pool, (uint64_t)Hkv * D, rows, (uint64_t)Hkv * D * 2, 64, (uint32_t)ps))) return rc;
+    a.page_table = page_table;
+    a.prefix = prefix_lens;
+    a.suffix = suffix_lens;
+    a.cu = s.cu;
+    a.units = s.units;
+    a.n_units = s.n_units;
+    a.err = err;
+    a.out = out;
+    a.num_pages = dims->num_pages;
+    a.Hq = Hq;
+    a.G = G;
+    a.ps = ps;
+    a.max_pages = dims->max_pages;
+    a.tq = tq;
+    a.oob_row = (int32_t)rows;
+    const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)D);
+    a.scale_log2 = scale * 1.4426950408889634f;
+    const int64_t grid = std::min<int64_t>((int64_t)sm_count, max_units);
+    e = rr::launch_extend_attention(a, D, (int)std::max<int64_t>(grid, 1), stream);
+    if (e != cudaSuccess) return cuda_fail(e, "extend attention kernel launch");
+    return RR_OK;
+}
