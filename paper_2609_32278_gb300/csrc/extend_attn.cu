@@ -54,7 +54,7 @@ constexpr int kWarpProducer = 8;
 constexpr int kWarpMMA = 9;
 constexpr long long kWaitLimitCycles = 1ll << 33;  // ~4 s at 2 GHz
 
-template <int D, int NS>
+template <int D, int NK, int NV>
 struct Cfg {
     static constexpr int kChunks = D / 64;                 // 128-byte (64 x bf16) column chunks
     static constexpr int kChunkBytes = kBM * 128;          // one chunk of a 128-row tile: 16 KiB
@@ -62,12 +62,12 @@ struct Cfg {
     static constexpr int kKVTileBytes = kBN * D * 2;
     static constexpr int kOffQ = 0;
     static constexpr int kOffK = kOffQ + kNQ * kQTileBytes;
-    static constexpr int kOffV = kOffK + NS * kKVTileBytes;
-    static constexpr int kOffBar = kOffV + NS * kKVTileBytes;
+    static constexpr int kOffV = kOffK + NK * kKVTileBytes;
+    static constexpr int kOffBar = kOffV + NV * kKVTileBytes;
     // barrier indices
     static constexpr int kQFull = 0, kQEmpty = 1;
-    static constexpr int kKFull = 2, kKEmpty = 2 + NS, kVFull = 2 + 2 * NS, kVEmpty = 2 + 3 * NS;
-    static constexpr int kSFull = 2 + 4 * NS, kPFull = kSFull + kNQ, kOFinal = kPFull + kNQ;
+    static constexpr int kKFull = 2, kKEmpty = 2 + NK, kVFull = 2 + 2 * NK, kVEmpty = 2 + 2 * NK + NV;
+    static constexpr int kSFull = 2 + 2 * NK + 2 * NV, kPFull = kSFull + kNQ, kOFinal = kPFull + kNQ;
     static constexpr int kVTmp = kOFinal + kNQ, kDrain = kVTmp + 1;
     static constexpr int kNumBars = kDrain + 1;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // u32 TMEM base, i32 abort flag
@@ -83,18 +83,18 @@ struct Ctl {
 };
 
 // Bounded wait on an mbarrier phase.  False: timed out (flag raised) or another role aborted.
+// Each try may suspend the thread (up to 0.2 ms) until the phase completes, so waiting
+// warps leave the issue slots to the warps that are computing.
 __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, const Ctl& c) {
     if (ptx::mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
-    for (uint32_t n = 1;; ++n) {
-        if (ptx::mbar_try_wait(bar, parity)) return true;
-        if ((n & 63) == 0) {
-            if (*c.abort_flag) return false;
-            if (clock64() - t0 > kWaitLimitCycles) {
-                *c.abort_flag = 1;
-                atomicCAS(c.err, 0, RR_ERR_TIMEOUT);
-                return false;
-            }
+    for (;;) {
+        if (ptx::mbar_try_wait_sleep(bar, parity, 200000u)) return true;
+        if (*c.abort_flag) return false;
+        if (clock64() - t0 > kWaitLimitCycles) {
+            *c.abort_flag = 1;
+            atomicCAS(c.err, 0, RR_ERR_TIMEOUT);
+            return false;
         }
     }
 }
@@ -112,9 +112,9 @@ __device__ __forceinline__ int unit_of(int wave, int cta, int grid) {
     return wave * grid + ((wave & 1) ? (grid - 1 - cta) : cta);
 }
 
-template <int D, int NS>
+template <int D, int NK, int NV, bool kPVFirst>
 __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_constant__ AttnArgs a) {
-    using C = Cfg<D, NS>;
+    using C = Cfg<D, NK, NV>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const uint32_t sb = ptx::smem_u32(smem);
@@ -127,9 +127,11 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
     if (threadIdx.x == 0) {
         ptx::mbar_init(bar(C::kQFull), 1);
         ptx::mbar_init(bar(C::kQEmpty), 1);
-        for (int s = 0; s < NS; ++s) {
+        for (int s = 0; s < NK; ++s) {
             ptx::mbar_init(bar(C::kKFull + s), 1);
             ptx::mbar_init(bar(C::kKEmpty + s), 1);
+        }
+        for (int s = 0; s < NV; ++s) {
             ptx::mbar_init(bar(C::kVFull + s), 1);
             ptx::mbar_init(bar(C::kVEmpty + s), 1);
         }
@@ -193,8 +195,8 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             if (!ok) break;
             const int last_page_end = ((n_keys + a.ps - 1) / a.ps) * a.ps;
             for (int j = 0; j < n_kv; ++j, ++kv_count) {
-                const int s = (int)(kv_count % NS);
-                const uint32_t use = kv_count / NS;
+                const int sk = (int)(kv_count % NK), sv = (int)(kv_count % NV);
+                const uint32_t usek = kv_count / NK, usev = kv_count / NV;
                 int row = a.oob_row;  // page past the agent's keys: zero fill
                 if (lane < ppt) {
                     const int lp = j * ppt + lane;
@@ -206,30 +208,30 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                 }
                 // K tile
                 if (lane == 0) {
-                    if (use > 0) ok = wait_bar(bar(C::kKEmpty + s), (use - 1) & 1, ctl);
-                    if (ok) ptx::mbar_arrive_expect_tx(bar(C::kKFull + s), C::kKVTileBytes);
+                    if (usek > 0) ok = wait_bar(bar(C::kKEmpty + sk), (usek - 1) & 1, ctl);
+                    if (ok) ptx::mbar_arrive_expect_tx(bar(C::kKFull + sk), C::kKVTileBytes);
                 }
                 ok = __shfl_sync(0xffffffffu, ok, 0);
                 if (!ok) break;
-                armed_k |= 1u << s;
-                par_k = (par_k & ~(1u << s)) | ((use & 1u) << s);
+                armed_k |= 1u << sk;
+                par_k = (par_k & ~(1u << sk)) | ((usek & 1u) << sk);
                 if (lane < ppt)
                     for (int c = 0; c < C::kChunks; ++c)
-                        ptx::tma_load_2d(sb + C::kOffK + s * C::kKVTileBytes + c * C::kChunkBytes + lane * a.ps * 128,
-                                         &a.tm_k, g * D + c * 64, row, bar(C::kKFull + s));
+                        ptx::tma_load_2d(sb + C::kOffK + sk * C::kKVTileBytes + c * C::kChunkBytes + lane * a.ps * 128,
+                                         &a.tm_k, g * D + c * 64, row, bar(C::kKFull + sk));
                 // V tile; if the agent's last page is only partly its own, land it on the
                 // side barrier, clear the foreign slots, then release it to the MMA warp.
                 const bool clear_tail = (j == n_kv - 1) && (last_page_end > agent_len);
-                const uint32_t vbar = clear_tail ? bar(C::kVTmp) : bar(C::kVFull + s);
+                const uint32_t vbar = clear_tail ? bar(C::kVTmp) : bar(C::kVFull + sv);
                 if (lane == 0) {
-                    if (use > 0) ok = wait_bar(bar(C::kVEmpty + s), (use - 1) & 1, ctl);
+                    if (usev > 0) ok = wait_bar(bar(C::kVEmpty + sv), (usev - 1) & 1, ctl);
                     if (ok) ptx::mbar_arrive_expect_tx(vbar, C::kKVTileBytes);
                 }
                 ok = __shfl_sync(0xffffffffu, ok, 0);
                 if (!ok) break;
                 if (lane < ppt)
                     for (int c = 0; c < C::kChunks; ++c)
-                        ptx::tma_load_2d(sb + C::kOffV + s * C::kKVTileBytes + c * C::kChunkBytes + lane * a.ps * 128,
+                        ptx::tma_load_2d(sb + C::kOffV + sv * C::kKVTileBytes + c * C::kChunkBytes + lane * a.ps * 128,
                                          &a.tm_v, g * D + c * 64, row, vbar);
                 if (clear_tail) {
                     armed_vtmp = (int)vtmp_phase;
@@ -239,17 +241,17 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                     armed_vtmp = -1;
                     vtmp_phase ^= 1;
                     const int r0 = agent_len - j * kBN;  // 0 < r0 < kBN: first row past the agent
-                    uint8_t* vt = smem + C::kOffV + s * C::kKVTileBytes;
+                    uint8_t* vt = smem + C::kOffV + sv * C::kKVTileBytes;
                     for (int c = 0; c < C::kChunks; ++c) {
                         uint4* base = reinterpret_cast<uint4*>(vt + c * C::kChunkBytes);
                         for (int e = r0 * 8 + lane; e < kBN * 8; e += 32) base[e] = make_uint4(0u, 0u, 0u, 0u);
                     }
                     ptx::fence_proxy_async_smem();
                     __syncwarp();
-                    if (lane == 0) ptx::mbar_arrive(bar(C::kVFull + s));
+                    if (lane == 0) ptx::mbar_arrive(bar(C::kVFull + sv));
                 } else {
-                    armed_v |= 1u << s;
-                    par_v = (par_v & ~(1u << s)) | ((use & 1u) << s);
+                    armed_v |= 1u << sv;
+                    par_v = (par_v & ~(1u << sv)) | ((usev & 1u) << sv);
                 }
             }
             ++unit_i;
@@ -257,10 +259,10 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
         if (!ok && lane == 0) {  // abort: let every copy this warp started land before exit
             if (armed_q >= 0) drain_bar(bar(C::kQFull), (uint32_t)armed_q);
             if (armed_vtmp >= 0) drain_bar(bar(C::kVTmp), (uint32_t)armed_vtmp);
-            for (int s = 0; s < NS; ++s) {
+            for (int s = 0; s < NK; ++s)
                 if (armed_k >> s & 1u) drain_bar(bar(C::kKFull + s), par_k >> s & 1u);
+            for (int s = 0; s < NV; ++s)
                 if (armed_v >> s & 1u) drain_bar(bar(C::kVFull + s), par_v >> s & 1u);
-            }
         }
         __syncwarp();
     } else if (warp == kWarpMMA) {
@@ -300,40 +302,64 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                 if (!(ok = wait_bar(bar(C::kQFull), unit_i & 1, ctl))) break;
                 ptx::tc_fence_after();
                 {
-                    const int s = (int)(kv_count % NS);
-                    if (!(ok = wait_bar(bar(C::kKFull + s), (kv_count / NS) & 1, ctl))) break;
+                    const int sk = (int)(kv_count % NK);
+                    if (!(ok = wait_bar(bar(C::kKFull + sk), (kv_count / NK) & 1, ctl))) break;
                     ptx::tc_fence_after();
-                    issue_qk(0, s);
+                    issue_qk(0, sk);
                     ptx::mma_commit(bar(C::kSFull + 0));
-                    issue_qk(1, s);
+                    issue_qk(1, sk);
                     ptx::mma_commit(bar(C::kSFull + 1));
-                    ptx::mma_commit(bar(C::kKEmpty + s));
+                    ptx::mma_commit(bar(C::kKEmpty + sk));
                 }
                 for (int j = 0; j < n_kv && ok; ++j) {
                     const uint32_t cur = kv_count + j, nxt = cur + 1;
-                    const int s = (int)(cur % NS), s1 = (int)(nxt % NS);
+                    const int sv = (int)(cur % NV), sk1 = (int)(nxt % NK);
                     const bool more = j + 1 < n_kv;
-                    if (!(ok = wait_bar(bar(C::kVFull + s), (cur / NS) & 1, ctl))) break;
+                    if (!(ok = wait_bar(bar(C::kVFull + sv), (cur / NV) & 1, ctl))) break;
                     ptx::tc_fence_after();
+                    if constexpr (kPVFirst) {
+                        // PV_0(j), PV_1(j), S_0(j+1), S_1(j+1): no two adjacent MMAs touch the same TMEM columns
 #pragma unroll
-                    for (int q = 0; q < kNQ; ++q) {
-                        if (!(ok = wait_bar(bar(C::kPFull + q), (p_phase >> q) & 1u, ctl))) break;
-                        p_phase ^= 1u << q;
-                        ptx::tc_fence_after();
-                        issue_pv(q, s, j > 0);
-                        if (!more) ptx::mma_commit(bar(C::kOFinal + q));
-                        if (more) {
-                            if (q == 0) {
-                                if (!(ok = wait_bar(bar(C::kKFull + s1), (nxt / NS) & 1, ctl))) break;
-                                ptx::tc_fence_after();
-                            }
-                            issue_qk(q, s1);
-                            ptx::mma_commit(bar(C::kSFull + q));
-                            if (q == kNQ - 1) ptx::mma_commit(bar(C::kKEmpty + s1));
+                        for (int q = 0; q < kNQ; ++q) {
+                            if (!(ok = wait_bar(bar(C::kPFull + q), (p_phase >> q) & 1u, ctl))) break;
+                            p_phase ^= 1u << q;
+                            ptx::tc_fence_after();
+                            issue_pv(q, sv, j > 0);
+                            if (!more) ptx::mma_commit(bar(C::kOFinal + q));
                         }
+                        if (!ok) break;
+                        ptx::mma_commit(bar(C::kVEmpty + sv));
+                        if (more) {
+                            if (!(ok = wait_bar(bar(C::kKFull + sk1), (nxt / NK) & 1, ctl))) break;
+                            ptx::tc_fence_after();
+                            issue_qk(0, sk1);
+                            ptx::mma_commit(bar(C::kSFull + 0));
+                            issue_qk(1, sk1);
+                            ptx::mma_commit(bar(C::kSFull + 1));
+                            ptx::mma_commit(bar(C::kKEmpty + sk1));
+                        }
+                    } else {
+                        // PV_0(j), S_0(j+1), PV_1(j), S_1(j+1): one Q tile's MMAs overlap the other's softmax
+#pragma unroll
+                        for (int q = 0; q < kNQ; ++q) {
+                            if (!(ok = wait_bar(bar(C::kPFull + q), (p_phase >> q) & 1u, ctl))) break;
+                            p_phase ^= 1u << q;
+                            ptx::tc_fence_after();
+                            issue_pv(q, sv, j > 0);
+                            if (!more) ptx::mma_commit(bar(C::kOFinal + q));
+                            if (more) {
+                                if (q == 0) {
+                                    if (!(ok = wait_bar(bar(C::kKFull + sk1), (nxt / NK) & 1, ctl))) break;
+                                    ptx::tc_fence_after();
+                                }
+                                issue_qk(q, sk1);
+                                ptx::mma_commit(bar(C::kSFull + q));
+                                if (q == kNQ - 1) ptx::mma_commit(bar(C::kKEmpty + sk1));
+                            }
+                        }
+                        if (!ok) break;
+                        ptx::mma_commit(bar(C::kVEmpty + sv));
                     }
-                    if (!ok) break;
-                    ptx::mma_commit(bar(C::kVEmpty + s));
                 }
                 if (!ok) break;
                 ptx::mma_commit(bar(C::kQEmpty));
@@ -373,28 +399,45 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                 if (!(ok = wait_bar(bar(C::kSFull + q), s_phase, ctl))) break;
                 s_phase ^= 1;
                 ptx::tc_fence_after();
+                // S row in two halves: the second half's TMEM load overlaps the first half's max.
                 uint32_t sr[kBN];
-#pragma unroll
-                for (int c = 0; c < kBN; c += 32) ptx::tmem_ld32(t_s + c, *reinterpret_cast<uint32_t(*)[32]>(&sr[c]));
-                ptx::tmem_wait_ld();
+                auto chunk = [&](int c) -> uint32_t(&)[32] { return *reinterpret_cast<uint32_t(*)[32]>(&sr[c]); };
+                ptx::tmem_ld32(t_s + 0, chunk(0));
+                ptx::tmem_ld32(t_s + 32, chunk(32));
+                ptx::tmem_wait_ld_regs(chunk(0));
+                ptx::tmem_wait_ld_regs(chunk(32));
+                ptx::tmem_ld32(t_s + 64, chunk(64));
+                ptx::tmem_ld32(t_s + 96, chunk(96));
                 float sv[kBN];
+                const bool masked = j >= mask_from;
+                const int lim = row_limit - j * kBN;  // columns past lim are invisible to this row
+                float mx[8];
 #pragma unroll
-                for (int c = 0; c < kBN; ++c) sv[c] = __uint_as_float(sr[c]);
-                if (j >= mask_from) {
-                    const int lim = row_limit - j * kBN;
+                for (int h = 0; h < 2; ++h) {
+                    if (h == 1) {
+                        ptx::tmem_wait_ld_regs(chunk(64));
+                        ptx::tmem_wait_ld_regs(chunk(96));
+                    }
 #pragma unroll
-                    for (int c = 0; c < kBN; ++c)
-                        if (c > lim) sv[c] = -INFINITY;
+                    for (int c = h * 64; c < h * 64 + 64; ++c) sv[c] = __uint_as_float(sr[c]);
+                    if (masked) {  // only the last tile or two of a unit
+#pragma unroll
+                        for (int c = h * 64; c < h * 64 + 64; ++c)
+                            if (c > lim) sv[c] = -INFINITY;
+                    }
+                    // eight independent chains of 3-input max over this half
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) {
+                        const int c = h * 64 + k * 8;
+                        float m = ptx::max3(sv[c], sv[c + 1], sv[c + 2]);
+                        m = ptx::max3(m, sv[c + 3], sv[c + 4]);
+                        m = ptx::max3(m, sv[c + 5], sv[c + 6]);
+                        m = h == 0 ? fmaxf(m, sv[c + 7]) : ptx::max3(m, sv[c + 7], mx[k]);
+                        mx[k] = m;
+                    }
                 }
-                float mx0 = sv[0], mx1 = sv[1], mx2 = sv[2], mx3 = sv[3];
-#pragma unroll
-                for (int c = 4; c < kBN; c += 4) {
-                    mx0 = fmaxf(mx0, sv[c]);
-                    mx1 = fmaxf(mx1, sv[c + 1]);
-                    mx2 = fmaxf(mx2, sv[c + 2]);
-                    mx3 = fmaxf(mx3, sv[c + 3]);
-                }
-                const float mxs = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2;
+                const float mxs = ptx::max3(ptx::max3(mx[0], mx[1], mx[2]), ptx::max3(mx[3], mx[4], mx[5]),
+                                            fmaxf(mx[6], mx[7])) * sl2;
                 bool grow = false;
                 float f = 1.0f;
                 if (j == 0) {
@@ -406,19 +449,27 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                     m_run = mxs;
                 }
                 const float neg = -m_run;
-                float l0 = 0.f, l1 = 0.f;
+                // p = 2^(s * scale * log2e - m): packed FMA, ex2, packed accumulation over 8 chains
+                float la[4] = {0.f, 0.f, 0.f, 0.f}, lb[4] = {0.f, 0.f, 0.f, 0.f};
                 uint32_t pk[kBN / 2];
 #pragma unroll
                 for (int c = 0; c < kBN; c += 2) {
-                    const float p0 = ptx::ex2_approx(fmaf(sv[c], sl2, neg));
-                    const float p1 = ptx::ex2_approx(fmaf(sv[c + 1], sl2, neg));
-                    l0 += p0;
-                    l1 += p1;
+                    float x0, x1;
+                    ptx::fma2(x0, x1, sv[c], sv[c + 1], sl2, sl2, neg, neg);
+                    const float p0 = ptx::ex2_approx(x0);
+                    const float p1 = ptx::ex2_approx(x1);
+                    const int k = (c >> 1) & 3;
+                    ptx::add2(la[k], lb[k], la[k], lb[k], p0, p1);
                     pk[c >> 1] = ptx::pack_bf16x2(p0, p1);
+                    if (c == kBN / 2 - 2) ptx::tmem_st32(t_s, *reinterpret_cast<uint32_t(*)[32]>(&pk[0]));
                 }
-                l_run += l0 + l1;
-                ptx::tmem_st32(t_s, *reinterpret_cast<uint32_t(*)[32]>(&pk[0]));
                 ptx::tmem_st32(t_s + 32, *reinterpret_cast<uint32_t(*)[32]>(&pk[32]));
+                {
+                    float s0, s1, s2, s3;
+                    ptx::add2(s0, s1, la[0], lb[0], la[1], lb[1]);
+                    ptx::add2(s2, s3, la[2], lb[2], la[3], lb[3]);
+                    l_run += (s0 + s2) + (s1 + s3);
+                }
                 // O_q holds PV of tiles < j (complete: S_q(j) was issued after PV_q(j-1)); bring it to the
                 // new max before PV_q(j) may start, i.e. before this thread signals P_q(j).
                 if (__any_sync(0xffffffffu, grow)) {  // warp-uniform: tcgen05.ld/st are .sync.aligned
@@ -426,7 +477,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                     for (int c = 0; c < D; c += 32) {
                         uint32_t o[32];
                         ptx::tmem_ld32(t_o + c, o);
-                        ptx::tmem_wait_ld();
+                        ptx::tmem_wait_ld_regs(o);
 #pragma unroll
                         for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * f);
                         ptx::tmem_st32(t_o + c, o);
@@ -448,7 +499,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             for (int c = 0; c < D; c += 32) {
                 uint32_t o[32];
                 ptx::tmem_ld32(t_o + c, o);
-                ptx::tmem_wait_ld();
+                ptx::tmem_wait_ld_regs(o);
                 uint32_t pk[16];
 #pragma unroll
                 for (int i = 0; i < 16; ++i)
@@ -470,35 +521,35 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
     }
 }
 
-template <int D, int NS>
+template <int D, int NK, int NV, bool kPVFirst>
 cudaError_t launch_cfg(const AttnArgs& a, int grid, cudaStream_t st) {
-    using C = Cfg<D, NS>;
+    using C = Cfg<D, NK, NV>;
     static bool attr_done[64] = {};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     if (!attr_done[dev]) {
-        e = cudaFuncSetAttribute(extend_attn_kernel<D, NS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(extend_attn_kernel<D, NK, NV, kPVFirst>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  C::kSmemBytes);
         if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
-    extend_attn_kernel<D, NS><<<grid, kThreads, C::kSmemBytes, st>>>(a);
+    extend_attn_kernel<D, NK, NV, kPVFirst><<<grid, kThreads, C::kSmemBytes, st>>>(a);
     return cudaGetLastError();
 }
 
 }  // namespace
 
 size_t extend_attention_smem_bytes(int head_dim) {
-    if (head_dim == 128) return Cfg<128, 2>::kSmemBytes;
-    if (head_dim == 64) return Cfg<64, 4>::kSmemBytes;
+    if (head_dim == 128) return Cfg<128, 2, 2>::kSmemBytes;
+    if (head_dim == 64) return Cfg<64, 4, 4>::kSmemBytes;
     return 0;
 }
 
 cudaError_t launch_extend_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st) {
-    if (head_dim == 128) return launch_cfg<128, 2>(a, grid, st);
-    if (head_dim == 64) return launch_cfg<64, 4>(a, grid, st);
+    if (head_dim == 128) return launch_cfg<128, 2, 2, false>(a, grid, st);
+    if (head_dim == 64) return launch_cfg<64, 4, 4, false>(a, grid, st);
     return cudaErrorInvalidValue;
 }
 
