@@ -237,6 +237,39 @@ def load_traffic(src_hash):
     return rec, rec
 
 
+def per_agent_latency(rr, wl, g, dev, st, reps=5):
+    """Each agent's extend step (append + attention) run alone, as a returning request would be.
+
+    The kernel-level analogue of per-request time to first token: RR-Evict trades a few whole-history
+    recomputes (LRU) for many partial ones, which shows up as a lower maximum here (Sec. 3.3, Sec. 4).
+    """
+    import torch
+    cu = wl.cu
+    times = []
+    for b in range(wl.B):
+        if wl.suffix_lens[b] == 0:
+            continue
+        r0, r1 = int(cu[b]), int(cu[b + 1])
+        args_b = (g["page_table"][b:b + 1], g["prefix_lens"][b:b + 1], g["suffix_lens"][b:b + 1])
+        out = g["out"][r0:r1]
+        ts = []
+        for k in range(reps + 1):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(st)
+            rr.kv_append(g["k_new"][r0:r1], g["v_new"][r0:r1], g["k_pool"], g["v_pool"], *args_b)
+            rr.extend_attention(g["q"][r0:r1], g["k_pool"], g["v_pool"], *args_b, out=out)
+            e1.record(st)
+            torch.cuda.synchronize(dev)
+            if k:
+                ts.append(e0.elapsed_time(e1))
+        times.append(statistics.median(ts))
+    if rr.device_error():
+        raise RuntimeError("device error in the per-agent leg")
+    t = np.array(times)
+    return {"agents": len(times), "max_ms": float(t.max()), "p99_ms": float(np.percentile(t, 99)),
+            "p50_ms": float(np.percentile(t, 50)), "mean_ms": float(t.mean()), "sum_ms": float(t.sum())}
+
+
 def run_ours(args, world, rank, local):
     import torch
     import synth
@@ -340,6 +373,10 @@ def run_ours(args, world, rank, local):
         e2e = {"value": world * F / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
 
+    per_agent = None
+    if args.per_agent:
+        per_agent = per_agent_latency(rr, wl, g, dev, st)
+
     achieved = F / (attn_ms * 1e-3) / 1e12
     src_hash = kernel_source_hash()
     traffic_rec, _ = load_traffic(src_hash)
@@ -371,6 +408,8 @@ def run_ours(args, world, rank, local):
         "gpu_launches": 4 * args.steps,
         "clocks": clk,
     }
+    if per_agent is not None:
+        line["per_agent_extend"] = per_agent
     if rank == 0 and not args.no_cpu_baseline:
         f, t, rows, threads = cpu_oracle_sample(wl, args.baseline_flops, seed=7)
         line["cpu_baseline"] = {"value": f / t / 1e12, "unit": "TFLOP/s", "cores": threads, "kind": "oracle",
@@ -393,6 +432,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--agents", type=int, default=0, help="only the first N agents (small profiling case)")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
+    ap.add_argument("--per-agent", action="store_true", help="also time each agent's extend step alone")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -122,13 +122,16 @@ int rr_extend_attention(const void* q, const void* k_pool, const void* v_pool, c
  * device-wide synchronisation of cudaMalloc/cudaFree.  This entry point
  * computes exactly what rr_extend_attention computes (same kernels, same
  * arguments and layouts), but keeps its schedule scratch in one fixed array
- * of static device memory (about 1.06 MiB) that every GPU loading the library
+ * of static device memory (about 1.31 MiB) that every GPU loading the library
  * holds until the process exits.  It calls no cudaMalloc, cudaFree or other
  * allocating routine.
  *
  * Limits: at most 4096 agents, and at most 65536 schedule work units, where
  * the units needed are bounded by Hkv * (T / (256 / G) + B + 1).  Larger
- * batches return RR_ERR_UNSUPPORTED without launching anything.
+ * batches return RR_ERR_UNSUPPORTED without launching anything.  It never
+ * splits a unit's key range across CTAs (that needs partial-result buffers),
+ * so small batches of long contexts run slower than through
+ * rr_extend_attention; results agree within the parity tolerance.
  *
  * device_error: optional device int32 (4-byte aligned) that receives a
  * device-side error code (RR_ERR_LENS, RR_ERR_OOB, RR_ERR_TIMEOUT) if one

@@ -174,7 +174,8 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             const int ui = unit_of(w, cta, grid);
             if (ui >= n_units) break;
             const int4 U = a.units[ui];
-            const int b = U.x, g = U.y, u = U.z, n_kv = U.w;
+            const int b = U.x, g = U.y & 0xFF, sp = (U.y >> 8) & 0xFF, ns = (U.y >> 16) & 0xFF, u = U.z;
+            const int n_kv = U.w, kb = sp * n_kv / ns, ke = (sp + 1) * n_kv / ns;  // this item's KV tiles
             const int P = a.prefix[b], S = a.suffix[b], cu_b = a.cu[b];
             const int t0 = u * unit_tokens;
             const int n_keys = P + min(S, t0 + unit_tokens);
@@ -194,7 +195,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             ok = __shfl_sync(0xffffffffu, ok, 0);
             if (!ok) break;
             const int last_page_end = ((n_keys + a.ps - 1) / a.ps) * a.ps;
-            for (int j = 0; j < n_kv; ++j, ++kv_count) {
+            for (int j = kb; j < ke; ++j, ++kv_count) {
                 const int sk = (int)(kv_count % NK), sv = (int)(kv_count % NV);
                 const uint32_t usek = kv_count / NK, usev = kv_count / NV;
                 int row = a.oob_row;  // page past the agent's keys: zero fill
@@ -298,7 +299,9 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             for (int w = 0; ok; ++w) {
                 const int ui = unit_of(w, cta, grid);
                 if (ui >= n_units) break;
-                const int n_kv = a.units[ui].w;
+                const int4 U = a.units[ui];
+                const int sp = (U.y >> 8) & 0xFF, ns = (U.y >> 16) & 0xFF;
+                const int n_kv = (sp + 1) * U.w / ns - sp * U.w / ns;  // KV tiles of this item
                 if (!(ok = wait_bar(bar(C::kQFull), unit_i & 1, ctl))) break;
                 ptx::tc_fence_after();
                 {
@@ -386,16 +389,15 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             const int ui = unit_of(w, cta, grid);
             if (ui >= n_units) break;
             const int4 U = a.units[ui];
-            const int b = U.x, g = U.y, u = U.z, n_kv = U.w;
-            const int P = a.prefix[b], S = a.suffix[b], cu_b = a.cu[b];
+            const int b = U.x, g = U.y & 0xFF, sp = (U.y >> 8) & 0xFF, ns = (U.y >> 16) & 0xFF, u = U.z;
+            const int kb = sp * U.w / ns, ke = (sp + 1) * U.w / ns;  // this item's KV tiles
+            const int P = a.prefix[b], agent_len = P + a.suffix[b];
             const int tq0 = u * unit_tokens + q * a.tq;  // first suffix token of this Q tile
             const int tok = tq0 + r / a.G;
-            const int head = g * a.G + r % a.G;
-            const int agent_len = P + S;
             const int row_limit = min(P + tok, agent_len - 1);     // last key this row may see
             const int mask_from = (min(P + tq0, agent_len - 1) + 1) / kBN;  // earlier tiles: no masking
             float m_run = -INFINITY, l_run = 0.f;
-            for (int j = 0; j < n_kv; ++j) {
+            for (int j = kb; j < ke; ++j) {
                 if (!(ok = wait_bar(bar(C::kSFull + q), s_phase, ctl))) break;
                 s_phase ^= 1;
                 ptx::tc_fence_after();
@@ -440,15 +442,15 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                                             fmaxf(mx[6], mx[7])) * sl2;
                 bool grow = false;
                 float f = 1.0f;
-                if (j == 0) {
-                    m_run = mxs;
+                if (j == kb) {
+                    m_run = mxs;  // -inf only for a row that sees no key of a later split's first tile
                 } else if (mxs > m_run + 8.0f) {
                     grow = true;
                     f = ptx::ex2_approx(m_run - mxs);
                     l_run *= f;
                     m_run = mxs;
                 }
-                const float neg = -m_run;
+                const float neg = m_run == -INFINITY ? 0.f : -m_run;  // a fully masked row stays at p = 0
                 // p = 2^(s * scale * log2e - m): packed FMA, ex2, packed accumulation over 8 chains
                 float la[4] = {0.f, 0.f, 0.f, 0.f}, lb[4] = {0.f, 0.f, 0.f, 0.f};
                 uint32_t pk[kBN / 2];
@@ -491,10 +493,29 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             if (!(ok = wait_bar(bar(C::kOFinal + q), o_phase, ctl))) break;
             o_phase ^= 1;
             ptx::tc_fence_after();
+            const int slot = a.item_slot[ui];
+            if (slot >= 0) {
+                // split item: unnormalised fp32 O row plus (max, sum); the combine kernel merges the splits
+                const long long prow = (long long)slot * (kNQ * kBM) + q * kBM + r;
+                float4* po = reinterpret_cast<float4*>(a.part_o + prow * D);
+#pragma unroll
+                for (int c = 0; c < D; c += 32) {
+                    uint32_t o[32];
+                    ptx::tmem_ld32(t_o + c, o);
+                    ptx::tmem_wait_ld_regs(o);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i)
+                        po[c / 4 + i] = make_float4(__uint_as_float(o[4 * i]), __uint_as_float(o[4 * i + 1]),
+                                                    __uint_as_float(o[4 * i + 2]), __uint_as_float(o[4 * i + 3]));
+                }
+                a.part_ml[prow] = make_float2(m_run, l_run);
+                continue;
+            }
             const float inv_l = 1.0f / l_run;
-            const bool valid = tok < S;
-            __nv_bfloat16* dst =
-                reinterpret_cast<__nv_bfloat16*>(a.out) + ((long long)(cu_b + tok) * a.Hq + head) * D;
+            const int tok_e = u * unit_tokens + q * a.tq + r / a.G;  // recomputed: keeps the tile loop lean
+            const bool valid = tok_e < a.suffix[b];
+            __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(a.out) +
+                                 ((long long)(a.cu[b] + tok_e) * a.Hq + g * a.G + r % a.G) * D;
 #pragma unroll
             for (int c = 0; c < D; c += 32) {
                 uint32_t o[32];

@@ -205,6 +205,18 @@ __device__ __forceinline__ void tmem_wait_ld_regs(uint32_t (&r)[32]) {
         : "memory");
 }
 
+// Warpgroup register reallocation: every warp of a warpgroup executes the same
+// one.  inc waits until enough registers have been released by a dec elsewhere in
+// the CTA, so the releasing warpgroup must run its dec unconditionally.
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_inc() {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_dec() {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
+}
+
 // ---------------------------------------------------------------- math
 
 // Three-input maximum (sm_100+).

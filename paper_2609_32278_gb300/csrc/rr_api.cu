@@ -2,6 +2,7 @@
 // the per-device workspace, TMA tensor-map encoding and kernel launches.
 #include <cstdarg>
 #include <cstdio>
+#include <algorithm>
 #include <cstring>
 #include <mutex>
 #include <vector>
@@ -43,17 +44,22 @@ PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
-// Workspace layout: [n_units, lens_ok][cu: B+1][unit_off: B+1][units: max_units x int4]
+// Workspace layout: [n_units, lens_ok, n_split][cu: B+1][unit_off: B+1][items: max_items x int4]
+// [item_slot: max_items][split units: max_split x int4][part_ml: slots x 256 float2][part_o: slots x 256 x D]
 struct Layout {
-    size_t off_cu, off_unit_off, off_units, total;
+    size_t off_cu, off_unit_off, off_units, off_slot, off_split, off_ml, off_o, total;
 };
 
-Layout layout_for(int64_t B, int64_t max_units) {
+Layout layout_for(int64_t B, int64_t max_items, int64_t max_split = 0, int64_t slots = 0, int64_t D = 0) {
     Layout L;
     L.off_cu = 256;
     L.off_unit_off = L.off_cu + align256((size_t)(B + 1) * 4);
     L.off_units = L.off_unit_off + align256((size_t)(B + 1) * 4);
-    L.total = L.off_units + align256((size_t)max_units * 16);
+    L.off_slot = L.off_units + align256((size_t)max_items * 16);
+    L.off_split = L.off_slot + align256((size_t)max_items * 4);
+    L.off_ml = L.off_split + align256((size_t)max_split * 16);
+    L.off_o = L.off_ml + align256((size_t)slots * rr::kNQ * rr::kBM * 8);
+    L.total = L.off_o + align256((size_t)slots * rr::kNQ * rr::kBM * (size_t)D * 4);
     return L;
 }
 
@@ -202,6 +208,10 @@ int rr_kv_append(const void* k_new, const void* v_new, void* k_pool, void* v_poo
     s.cu = reinterpret_cast<int32_t*>(ws + L.off_cu);
     s.unit_off = reinterpret_cast<int32_t*>(ws + L.off_unit_off);
     s.units = nullptr;
+    s.item_slot = nullptr;
+    s.split_units = nullptr;
+    s.n_split = reinterpret_cast<int32_t*>(ws) + 2;
+    s.split_grid = 0;
     s.n_units = reinterpret_cast<int32_t*>(ws);
     s.lens_ok = reinterpret_cast<int32_t*>(ws) + 1;
     s.err = d->err;
@@ -256,7 +266,14 @@ int rr_extend_attention(const void* q, const void* k_pool, const void* v_pool, c
     Device* d = nullptr;
     if ((rc = current_device(&d, nullptr))) return rc;
     if ((rc = get_encoder())) return rc;
-    const Layout L = layout_for(B, max_units);
+    // Split-K is possible only when the batch may have fewer than two waves of units; the batch has at
+    // least Hkv * T / unit_tokens units, so larger batches never split and need no partial buffers.
+    const int grid_sm = d->sm_count;
+    const bool may_split = (int64_t)Hkv * (T / unit_tokens) < 2ll * grid_sm;
+    const int64_t max_split = may_split ? 2ll * grid_sm : 0;
+    const int64_t slots = may_split ? 4ll * grid_sm : 0;
+    const int64_t max_items = std::max<int64_t>(max_units, slots);
+    const Layout L = layout_for(B, max_items, max_split, slots, D);
     if ((rc = ensure_ws(*d, L.total))) return rc;
     uint8_t* ws = static_cast<uint8_t*>(d->ws);
 
@@ -274,6 +291,10 @@ int rr_extend_attention(const void* q, const void* k_pool, const void* v_pool, c
     s.cu = reinterpret_cast<int32_t*>(ws + L.off_cu);
     s.unit_off = reinterpret_cast<int32_t*>(ws + L.off_unit_off);
     s.units = reinterpret_cast<int4*>(ws + L.off_units);
+    s.item_slot = reinterpret_cast<int32_t*>(ws + L.off_slot);
+    s.split_units = reinterpret_cast<int4*>(ws + L.off_split);
+    s.n_split = reinterpret_cast<int32_t*>(ws) + 2;
+    s.split_grid = may_split ? grid_sm : 0;
     s.n_units = reinterpret_cast<int32_t*>(ws);
     s.lens_ok = reinterpret_cast<int32_t*>(ws) + 1;
     s.err = d->err;
@@ -295,6 +316,9 @@ int rr_extend_attention(const void* q, const void* k_pool, const void* v_pool, c
     a.cu = s.cu;
     a.units = s.units;
     a.n_units = s.n_units;
+    a.item_slot = s.item_slot;
+    a.part_o = reinterpret_cast<float*>(ws + L.off_o);
+    a.part_ml = reinterpret_cast<float2*>(ws + L.off_ml);
     a.err = d->err;
     a.out = out;
     a.num_pages = dims->num_pages;
@@ -306,9 +330,25 @@ int rr_extend_attention(const void* q, const void* k_pool, const void* v_pool, c
     a.oob_row = (int32_t)rows;
     const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)D);
     a.scale_log2 = scale * 1.4426950408889634f;
-    const int64_t grid = std::min<int64_t>((int64_t)d->sm_count, max_units);
+    const int64_t grid = std::min<int64_t>((int64_t)d->sm_count, max_items);
     e = rr::launch_extend_attention(a, D, (int)std::max<int64_t>(grid, 1), stream);
     if (e != cudaSuccess) return cuda_fail(e, "extend attention kernel launch");
+    if (may_split) {
+        rr::CombineArgs c;
+        c.split_units = s.split_units;
+        c.n_split = s.n_split;
+        c.part_o = a.part_o;
+        c.part_ml = a.part_ml;
+        c.suffix = suffix_lens;
+        c.cu = s.cu;
+        c.out = out;
+        c.Hq = Hq;
+        c.G = G;
+        c.D = D;
+        c.tq = tq;
+        e = rr::launch_combine(c, (int)max_split, stream);
+        if (e != cudaSuccess) return cuda_fail(e, "split-K combine kernel launch");
+    }
     return RR_OK;
 }
 
@@ -401,10 +441,11 @@ namespace {
 
 constexpr int32_t kNoAllocMaxBatch = 4096;    // agents per call
 constexpr int64_t kNoAllocMaxUnits = 65536;   // schedule work units per call
-constexpr size_t kNoAllocOffCu = 256;         // [0] n_units, [1] lens_ok, [2] spare error word
+constexpr size_t kNoAllocOffCu = 256;         // [0] n_units, [1] lens_ok, [2] spare error word, [3] n_split
 constexpr size_t kNoAllocOffUnitOff = kNoAllocOffCu + ((size_t)(kNoAllocMaxBatch + 1) * 4 + 255) / 256 * 256;
 constexpr size_t kNoAllocOffUnits = kNoAllocOffUnitOff + ((size_t)(kNoAllocMaxBatch + 1) * 4 + 255) / 256 * 256;
-constexpr size_t kNoAllocBytes = kNoAllocOffUnits + (size_t)kNoAllocMaxUnits * 16;  // ~1.06 MiB
+constexpr size_t kNoAllocOffSlot = kNoAllocOffUnits + (size_t)kNoAllocMaxUnits * 16;
+constexpr size_t kNoAllocBytes = kNoAllocOffSlot + (size_t)kNoAllocMaxUnits * 4;  // ~1.31 MiB
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
 
@@ -494,6 +535,10 @@ extern "C" int rr_extend_attention_noalloc(const void* q, const void* k_pool, co
     s.cu = reinterpret_cast<int32_t*>(ws + kNoAllocOffCu);
     s.unit_off = reinterpret_cast<int32_t*>(ws + kNoAllocOffUnitOff);
     s.units = reinterpret_cast<int4*>(ws + kNoAllocOffUnits);
+    s.item_slot = reinterpret_cast<int32_t*>(ws + kNoAllocOffSlot);
+    s.split_units = nullptr;                       // no split-K: the partial buffers would not fit
+    s.n_split = reinterpret_cast<int32_t*>(ws) + 3;
+    s.split_grid = 0;
     s.n_units = reinterpret_cast<int32_t*>(ws);
     s.lens_ok = reinterpret_cast<int32_t*>(ws) + 1;
     s.err = err;
@@ -515,6 +560,9 @@ extern "C" int rr_extend_attention_noalloc(const void* q, const void* k_pool, co
     a.cu = s.cu;
     a.units = s.units;
     a.n_units = s.n_units;
+    a.item_slot = s.item_slot;
+    a.part_o = nullptr;
+    a.part_ml = nullptr;
     a.err = err;
     a.out = out;
     a.num_pages = dims->num_pages;

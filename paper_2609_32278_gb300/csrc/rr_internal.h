@@ -27,8 +27,13 @@ struct SchedArgs {
     int32_t build_units;   // 0: lengths prefix sums only (append)
     int32_t* cu;           // [B+1] exclusive prefix sum of suffix lens
     int32_t* unit_off;     // [B+1] first work unit of each agent
-    int4* units;           // [max_units] (agent, kv head, unit index, KV tiles), most expensive first
-    int32_t* n_units;
+    int4* units;           // [max_items] (agent, kv head | split << 8 | nsplit << 16, unit, KV tiles of the unit),
+                           // most expensive first
+    int32_t* item_slot;    // [max_items] partial-result slot of a split item, -1 if the unit is not split
+    int4* split_units;     // [units] split units for the combine: (agent, kv head | nsplit << 16, unit, first slot)
+    int32_t* n_split;      // number of split units
+    int32_t split_grid;    // persistent grid size; 0 disables splitting
+    int32_t* n_units;      // number of items
     int32_t* lens_ok;
     int32_t* err;
 };
@@ -59,6 +64,9 @@ struct AttnArgs {
     const int32_t* cu;
     const int4* units;
     const int32_t* n_units;
+    const int32_t* item_slot;  // partial-result slot of each item (-1: not split, write out directly)
+    float* part_o;         // [slots][kNQ * kBM][D] fp32 unnormalised partial outputs of split items
+    float2* part_ml;       // [slots][kNQ * kBM] (running max in log2 units, sum of weights)
     int32_t* err;
     void* out;             // [T][Hq][D] bf16
     int64_t num_pages;
@@ -68,7 +76,19 @@ struct AttnArgs {
     float scale_log2;      // softmax scale * log2(e)
 };
 
+struct CombineArgs {
+    const int4* split_units;  // (agent, kv head | nsplit << 16, unit, first slot)
+    const int32_t* n_split;
+    const float* part_o;
+    const float2* part_ml;
+    const int32_t* suffix;
+    const int32_t* cu;
+    void* out;
+    int32_t Hq, G, D, tq;
+};
+
 cudaError_t launch_sched(const SchedArgs& a, cudaStream_t st);
+cudaError_t launch_combine(const CombineArgs& a, int grid, cudaStream_t st);
 cudaError_t launch_kv_append(const AppendArgs& a, int sm_count, cudaStream_t st);
 // Returns cudaErrorInvalidValue for an unsupported head dim.
 cudaError_t launch_extend_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st);

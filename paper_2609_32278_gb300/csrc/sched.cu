@@ -7,7 +7,10 @@
 //   2. (attention only) give every work unit -- one KV head of one agent,
 //      kNQ consecutive Q tiles of its suffix -- its cost in KV tiles, the
 //      number of 128-key tiles its last row must read (prefix + covered suffix);
-//   3. counting-sort the units by cost, most expensive first, so a persistent
+//   3. if the batch has fewer than two waves of units, split each unit's KV
+//      range into items (split-K) so the grid stays full; the partial results
+//      are merged by the combine kernel;
+//   4. counting-sort the items by cost, most expensive first, so a persistent
 //      grid that takes them in order approximates longest-processing-time
 //      scheduling.  This is what balances a batch whose agents have very
 //      different cached prefixes and uncached suffixes (the skew an eviction
@@ -28,6 +31,54 @@ __device__ __forceinline__ int last_le(const int32_t* off, int n, long long x) {
         if ((long long)off[mid] <= x) lo = mid; else hi = mid - 1;
     }
     return lo;
+}
+
+// Sum over the 1024 threads of the block (every thread gets the total).
+__device__ long long block_sum(long long v, long long* s_ws) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    __syncthreads();
+    if (lane == 0) s_ws[warp] = v;
+    __syncthreads();
+    long long t = 0;
+#pragma unroll 4
+    for (int w = 0; w < 32; ++w) t += s_ws[w];
+    __syncthreads();
+    return t;
+}
+
+// Block-wide exclusive prefix sums of two values at once, in thread order; also returns the totals.
+__device__ void block_exclusive_scan2(long long x, long long y, long long& ex, long long& ey, long long& tx,
+                                      long long& ty, long long* s_wx, long long* s_wy) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    long long ix = x, iy = y;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const long long px = __shfl_up_sync(0xffffffffu, ix, o);
+        const long long py = __shfl_up_sync(0xffffffffu, iy, o);
+        if (lane >= o) { ix += px; iy += py; }
+    }
+    __syncthreads();
+    if (lane == 31) { s_wx[warp] = ix; s_wy[warp] = iy; }
+    __syncthreads();
+    if (warp == 0) {
+        long long wx = s_wx[lane], wy = s_wy[lane];
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const long long px = __shfl_up_sync(0xffffffffu, wx, o);
+            const long long py = __shfl_up_sync(0xffffffffu, wy, o);
+            if (lane >= o) { wx += px; wy += py; }
+        }
+        s_wx[lane] = wx;
+        s_wy[lane] = wy;
+    }
+    __syncthreads();
+    ex = (warp ? s_wx[warp - 1] : 0) + ix - x;
+    ey = (warp ? s_wy[warp - 1] : 0) + iy - y;
+    tx = s_wx[31];
+    ty = s_wy[31];
+    __syncthreads();
 }
 
 __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
@@ -98,22 +149,64 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     if (tid == 0) *a.lens_ok = 1;
     if (!a.build_units) return;
 
-    // ---- 2. histogram of unit costs
-    for (int i = tid; i < kCostBuckets; i += 1024) s_hist[i] = 0;
-    __syncthreads();  // also publishes cu / unit_off written above to the whole block
+    // ---- 2. unit costs and their total (the split decision needs it)
+    long long my_cost = 0;
     for (long long idx = tid; idx < tot_u; idx += 1024) {
         const int b = last_le(a.unit_off, B, idx);
         const int S = a.suffix[b], P = a.prefix[b];
         const int nu = (S + a.unit_tokens - 1) / a.unit_tokens;
-        const int local = (int)(idx - a.unit_off[b]);
-        const int u = local % nu;
+        const int u = (int)(idx - a.unit_off[b]) % nu;
         const long long n_keys = (long long)P + min((long long)S, (long long)(u + 1) * a.unit_tokens);
-        const long long cost = (n_keys + kBN - 1) / kBN;
-        atomicAdd(&s_hist[(int)min(cost, (long long)kCostBuckets - 1)], 1);
+        my_cost += (n_keys + kBN - 1) / kBN;
+    }
+    const long long tot_cost = block_sum(my_cost, s_ws);
+
+    // Split the KV range of every unit when the batch has fewer than two waves of units: a unit of
+    // `cost` KV tiles becomes ceil(cost / target) items (at most 64), target = total / (2 waves), at
+    // least 8 tiles.  Then items <= total/target + units <= 4 waves, which bounds the partial buffers.
+    const bool split = a.split_grid > 0 && tot_u < 2ll * a.split_grid && tot_u <= 1024 && tot_u > 0;
+    const long long target = split ? max(8ll, (tot_cost + 2ll * a.split_grid - 1) / (2ll * a.split_grid)) : 0;
+    int my_b = 0, my_g = 0, my_u = 0, my_ns = 1;
+    long long my_unit_cost = 0;
+    if (split && tid < tot_u) {  // one unit per thread
+        my_b = last_le(a.unit_off, B, tid);
+        const int S = a.suffix[my_b], P = a.prefix[my_b];
+        const int nu = (S + a.unit_tokens - 1) / a.unit_tokens;
+        const int local = tid - a.unit_off[my_b];
+        my_g = local / nu;
+        my_u = local % nu;
+        const long long n_keys = (long long)P + min((long long)S, (long long)(my_u + 1) * a.unit_tokens);
+        my_unit_cost = (n_keys + kBN - 1) / kBN;
+        my_ns = (int)min(min(64ll, my_unit_cost), (my_unit_cost + target - 1) / target);
+        if (my_ns < 1) my_ns = 1;
+    }
+    // partial-result slots and the rank of each split unit (exclusive scans over units)
+    long long my_slot_base = 0, my_rank = 0, n_slots = 0, n_split_units = 0;
+    block_exclusive_scan2(my_ns > 1 ? my_ns : 0, my_ns > 1 ? 1 : 0, my_slot_base, my_rank, n_slots, n_split_units,
+                          s_ws, s_wu);
+
+    // ---- 3. histogram of item costs
+    for (int i = tid; i < kCostBuckets; i += 1024) s_hist[i] = 0;
+    __syncthreads();
+    if (!split) {
+        for (long long idx = tid; idx < tot_u; idx += 1024) {
+            const int b = last_le(a.unit_off, B, idx);
+            const int S = a.suffix[b], P = a.prefix[b];
+            const int nu = (S + a.unit_tokens - 1) / a.unit_tokens;
+            const int u = (int)(idx - a.unit_off[b]) % nu;
+            const long long n_keys = (long long)P + min((long long)S, (long long)(u + 1) * a.unit_tokens);
+            const long long cost = (n_keys + kBN - 1) / kBN;
+            atomicAdd(&s_hist[(int)min(cost, (long long)kCostBuckets - 1)], 1);
+        }
+    } else if (tid < tot_u) {
+        for (int sp = 0; sp < my_ns; ++sp) {
+            const long long c = (sp + 1) * my_unit_cost / my_ns - sp * my_unit_cost / my_ns;
+            atomicAdd(&s_hist[(int)min(c, (long long)kCostBuckets - 1)], 1);
+        }
     }
     __syncthreads();
 
-    // ---- 3. exclusive scan in descending cost order: start[k] = sum of hist[k'] for k' > k
+    // ---- 4. exclusive scan in descending cost order: start[k] = sum of hist[k'] for k' > k
     {
         constexpr int kPer = kCostBuckets / 1024;
         int v[kPer];
@@ -123,27 +216,9 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
             v[i] = s_hist[kCostBuckets - 1 - (tid * kPer + i)];
             local += v[i];
         }
-        int inc = local;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            int y = __shfl_up_sync(0xffffffffu, inc, o);
-            if (lane >= o) inc += y;
-        }
-        __syncthreads();
-        if (lane == 31) s_ws[warp] = inc;
-        __syncthreads();
-        if (warp == 0) {
-            long long x = s_ws[lane];
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                long long y = __shfl_up_sync(0xffffffffu, x, o);
-                if (lane >= o) x += y;
-            }
-            s_ws[lane] = x;
-        }
-        __syncthreads();
-        int run = (int)((warp ? s_ws[warp - 1] : 0) + inc - local);
-        __syncthreads();
+        long long ex = 0, dummy = 0, t0 = 0, t1 = 0;
+        block_exclusive_scan2(local, 0, ex, dummy, t0, t1, s_ws, s_wu);
+        int run = (int)ex;
 #pragma unroll
         for (int i = 0; i < kPer; ++i) {
             s_hist[kCostBuckets - 1 - (tid * kPer + i)] = run;  // becomes the bucket's cursor
@@ -152,19 +227,33 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     }
     __syncthreads();
 
-    // ---- 4. scatter
-    for (long long idx = tid; idx < tot_u; idx += 1024) {
-        const int b = last_le(a.unit_off, B, idx);
-        const int S = a.suffix[b], P = a.prefix[b];
-        const int nu = (S + a.unit_tokens - 1) / a.unit_tokens;
-        const int local = (int)(idx - a.unit_off[b]);
-        const int h = local / nu, u = local % nu;
-        const long long n_keys = (long long)P + min((long long)S, (long long)(u + 1) * a.unit_tokens);
-        const long long cost = (n_keys + kBN - 1) / kBN;
-        const int pos = atomicAdd(&s_hist[(int)min(cost, (long long)kCostBuckets - 1)], 1);
-        a.units[pos] = make_int4(b, h, u, (int)cost);
+    // ---- 5. scatter: item = (agent, kv head | split << 8 | nsplit << 16, unit, KV tiles of the whole unit)
+    if (!split) {
+        for (long long idx = tid; idx < tot_u; idx += 1024) {
+            const int b = last_le(a.unit_off, B, idx);
+            const int S = a.suffix[b], P = a.prefix[b];
+            const int nu = (S + a.unit_tokens - 1) / a.unit_tokens;
+            const int local = (int)(idx - a.unit_off[b]);
+            const int h = local / nu, u = local % nu;
+            const long long n_keys = (long long)P + min((long long)S, (long long)(u + 1) * a.unit_tokens);
+            const long long cost = (n_keys + kBN - 1) / kBN;
+            const int pos = atomicAdd(&s_hist[(int)min(cost, (long long)kCostBuckets - 1)], 1);
+            a.units[pos] = make_int4(b, h | (1 << 16), u, (int)cost);
+            a.item_slot[pos] = -1;
+        }
+    } else if (tid < tot_u) {
+        for (int sp = 0; sp < my_ns; ++sp) {
+            const long long c = (sp + 1) * my_unit_cost / my_ns - sp * my_unit_cost / my_ns;
+            const int pos = atomicAdd(&s_hist[(int)min(c, (long long)kCostBuckets - 1)], 1);
+            a.units[pos] = make_int4(my_b, my_g | (sp << 8) | (my_ns << 16), my_u, (int)my_unit_cost);
+            a.item_slot[pos] = my_ns > 1 ? (int)(my_slot_base + sp) : -1;
+        }
+        if (my_ns > 1) a.split_units[my_rank] = make_int4(my_b, my_g | (my_ns << 16), my_u, (int)my_slot_base);
     }
-    if (tid == 0) *a.n_units = (int32_t)tot_u;
+    if (tid == 0) {
+        *a.n_units = split ? (int32_t)(n_slots + (tot_u - n_split_units)) : (int32_t)tot_u;
+        *a.n_split = split ? (int32_t)n_split_units : 0;
+    }
 }
 
 }  // namespace
