@@ -6,7 +6,7 @@
 //
 //   out[cu_b+i, h, :] = softmax_j( scale * q[cu_b+i, h, :] . K_j ) V_j,  j = 0 .. P_b + i
 //
-// Design (one persistent CTA per SM, 10 warps):
+// Design (one persistent CTA per SM, 12 warps; warp 11 only lends its registers):
 //   * work unit = (agent b, KV head g, kNQ = 2 consecutive Q tiles).  A Q tile
 //     packs 128/G suffix tokens x the G query heads that share KV head g into
 //     128 rows (GQA packing), so each K/V tile is loaded once for the whole
@@ -21,7 +21,19 @@
 //     K-major, 128B swizzle) into TMEM, and O_q += P_q V (TS: P read from TMEM,
 //     V from shared memory as an MN-major operand).  Issue order per KV tile j:
 //     PV_0(j), S_0(j+1), PV_1(j), S_1(j+1): the tensor core works on one Q
-//     tile while the softmax warpgroup of the other runs.
+//     tile while the softmax warpgroup of the other runs, and a tile's PV and
+//     next S run back to back, which keeps that tile's softmax-to-softmax
+//     chain short.  (Two issuers, one per tile, were measured slower: the
+//     tensor core then interleaves both tiles' GEMMs and every chain doubles.)
+//     P_1(j) is tested with a non-blocking mbarrier.test_wait issued in the
+//     same asm block as the last two MMAs of S_0(j+1), so the test's latency
+//     hides behind them; the blocking wait runs only if the phase was open.
+//   * warp 10, stage watcher (one thread): waits until V(j) and K(j+1) have
+//     landed and adds one arrival to P_0(j), so the MMA issuer's wait for
+//     P_0(j) covers both.  A wait on an mbarrier, even one already complete,
+//     costs the issuing thread ~250 cycles while the tensor core is busy, and
+//     with an MMA queue about one instruction deep every such wait idles the
+//     tensor core; the issuer is left with one wait per Q tile and KV tile.
 //   * warps 0-3 / 4-7, softmax warpgroups for Q tile 0 / 1: thread r owns row
 //     r (= TMEM lane r).  It loads its S row from TMEM, applies the causal mask
 //     on the tiles that need it, keeps a running max in log2 units and rescales
@@ -29,7 +41,9 @@
 //     probability <= 256, far inside bf16/fp32 range), writes P as bf16 back
 //     over its S columns, and at the end of the unit normalises O and stores it.
 //   TMEM: S_0 cols 0-127, S_1 128-255, O_0 256.., O_1 256+D.. (512 allocated).
-//   Shared memory (D=128): Q 2 x 32 KiB, K and V 2 stages x 32 KiB each.
+//   Shared memory (D=128): Q 2 x 32 KiB, K 2 and V 3 stages of 32 KiB (the
+//   producer loads K(i), V(i) in order; a third V stage keeps it from stalling
+//   on V's stage while K(i+1)'s is already free).
 //
 // Ordering facts the pipeline relies on: tcgen05.mma operations issued by one
 // thread execute in order, and tcgen05.commit arrives only after every earlier
@@ -49,9 +63,16 @@ namespace rr {
 
 namespace {
 
-constexpr int kThreads = 320;
+constexpr int kThreads = 384;  // warpgroups: softmax Q tile 0, softmax Q tile 1, producer + MMA + stage (+1 idle)
+// Register split (launch: 384 threads x 168 = 64512; 3 warps per SMSP): the producer/MMA warpgroup
+// drops to kRegsControl and each softmax warpgroup rises to kRegsSoftmax.
+constexpr uint32_t kRegsSoftmax = 192;
+constexpr uint32_t kRegsControl = 112;
+static_assert(2 * 128 * kRegsSoftmax + 128 * kRegsControl <= kThreads * 168, "register split exceeds the launch");
+static_assert((2 * kRegsSoftmax + kRegsControl) * 32 <= 16384, "register split exceeds one SMSP's file");
 constexpr int kWarpProducer = 8;
 constexpr int kWarpMMA = 9;
+constexpr int kWarpStage = 10;
 constexpr long long kWaitLimitCycles = 1ll << 33;  // ~4 s at 2 GHz
 
 template <int D, int NK, int NV>
@@ -68,8 +89,8 @@ struct Cfg {
     static constexpr int kQFull = 0, kQEmpty = 1;
     static constexpr int kKFull = 2, kKEmpty = 2 + NK, kVFull = 2 + 2 * NK, kVEmpty = 2 + 2 * NK + NV;
     static constexpr int kSFull = 2 + 2 * NK + 2 * NV, kPFull = kSFull + kNQ, kOFinal = kPFull + kNQ;
-    static constexpr int kVTmp = kOFinal + kNQ, kDrain = kVTmp + 1;
-    static constexpr int kNumBars = kDrain + 1;
+    static constexpr int kVTmp = kOFinal + kNQ, kDrain = kVTmp + 1, kDone = kDrain + 1;
+    static constexpr int kNumBars = kDone + 1;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // u32 TMEM base, i32 abort flag
     static constexpr int kSmemBytes = kOffMisc + 16 + 1024;  // + slack to align the base to 1 KiB
     static_assert(kChunkBytes % 1024 == 0, "swizzle atoms must stay 1 KiB aligned");
@@ -107,12 +128,46 @@ __device__ __forceinline__ void drain_bar(uint32_t bar, uint32_t parity) {
     }
 }
 
+// 2^x for a pair of floats on the FMA pipe, taking part of the exponential load off the MUFU unit.
+// Range reduction: x is clamped to [-126, +inf) (the lazy-rescale bound keeps x <= 8) and rounded to
+// the nearest integer n by adding 1.5 * 2^23 (the sum's low mantissa bits then hold n, a standard
+// round-to-nearest technique); r = x - n lies in [-1/2, 1/2].  2^r is a cubic whose coefficients
+// were fitted to 2^r on [-1/2, 1/2] by iteratively reweighted least squares on Chebyshev nodes
+// (Lawson's algorithm towards the minimax relative error): max relative error 7.5e-5 (2^-13.7),
+// far inside the bf16 rounding (2^-9) that P gets next.  The exponent n is added to the result's
+// exponent field by integer addition of n << 23 (the bits of the rounded sum shifted left by 23).
+constexpr float kExp2C0 = 0.99992807f, kExp2C1 = 0.69326099f, kExp2C2 = 0.24261112f, kExp2C3 = 0.05517166f;
+constexpr float kRoundMagic = 12582912.0f;  // 1.5 * 2^23
+
+__device__ __forceinline__ void exp2_poly2(float& p0, float& p1, float x0, float x1) {
+    x0 = fmaxf(x0, -126.f);
+    x1 = fmaxf(x1, -126.f);
+    float y0, y1, t0, t1, r0, r1, q0, q1;
+    ptx::add2(y0, y1, x0, x1, kRoundMagic, kRoundMagic);
+    ptx::add2(t0, t1, y0, y1, -kRoundMagic, -kRoundMagic);
+    ptx::fma2(r0, r1, t0, t1, -1.f, -1.f, x0, x1);  // r = x - round(x)
+    ptx::fma2(q0, q1, r0, r1, kExp2C3, kExp2C3, kExp2C2, kExp2C2);
+    ptx::fma2(q0, q1, q0, q1, r0, r1, kExp2C1, kExp2C1);
+    ptx::fma2(q0, q1, q0, q1, r0, r1, kExp2C0, kExp2C0);
+    p0 = __int_as_float(__float_as_int(q0) + (__float_as_int(y0) << 23));
+    p1 = __int_as_float(__float_as_int(q1) + (__float_as_int(y1) << 23));
+}
+
+// Every kEmuPairStride-th pair of scores goes through exp2_poly2, the others through MUFU ex2
+// (0: MUFU only, the default: on GB300 the softmax is bound by instruction issue, not by the MUFU
+// unit -- measured 1314 TFLOP/s with no offload against 1260 / 1219 / 1204 for 1/8 / 1/4 / 1/3).
+
+#ifndef RR_EMU_PAIR_STRIDE
+#define RR_EMU_PAIR_STRIDE 0
+#endif
+constexpr int kEmuPairStride = RR_EMU_PAIR_STRIDE;
+
 // Snake order: even waves left to right, odd waves right to left.
 __device__ __forceinline__ int unit_of(int wave, int cta, int grid) {
     return wave * grid + ((wave & 1) ? (grid - 1 - cta) : cta);
 }
 
-template <int D, int NK, int NV, bool kPVFirst>
+template <int D, int NK, int NV>
 __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_constant__ AttnArgs a) {
     using C = Cfg<D, NK, NV>;
     extern __shared__ uint8_t smem_raw[];
@@ -137,11 +192,12 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
         }
         for (int q = 0; q < kNQ; ++q) {
             ptx::mbar_init(bar(C::kSFull + q), 1);
-            ptx::mbar_init(bar(C::kPFull + q), kBM);
+            ptx::mbar_init(bar(C::kPFull + q), q == 0 ? kBM + 1 : kBM);  // + the stage warp on P_0
             ptx::mbar_init(bar(C::kOFinal + q), 1);
         }
         ptx::mbar_init(bar(C::kVTmp), 1);
         ptx::mbar_init(bar(C::kDrain), 1);
+        ptx::mbar_init(bar(C::kDone), 2 * kBM);  // every softmax thread, once, at its end
         *abort_flag = 0;
         ptx::fence_mbar_init();
     }
@@ -162,6 +218,9 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
     const int grid = gridDim.x, cta = blockIdx.x;
     const int unit_tokens = kNQ * a.tq;
 
+    if (warp >= 8) {
+    // ================================================================ control warpgroup (warps 8-11)
+    ptx::setmaxnreg_dec<kRegsControl>();  // whole warpgroup, unconditionally: the softmax warpgroups wait for it
     if (warp == kWarpProducer) {
         // ------------------------------------------------------------ TMA producer
         const int ppt = kBN / a.ps;  // pages per KV tile (<= 16)
@@ -266,6 +325,30 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                 if (armed_v >> s & 1u) drain_bar(bar(C::kVFull + s), par_v >> s & 1u);
         }
         __syncwarp();
+    } else if (warp == kWarpStage) {
+        // ------------------------------------------------------------ stage watcher
+        if (lane == 0) {
+            uint32_t kv_count = 0, p_phase = 0;
+            bool ok = true;
+            for (int w = 0; ok; ++w) {
+                const int ui = unit_of(w, cta, grid);
+                if (ui >= n_units) break;
+                const int4 U = a.units[ui];
+                const int sp = (U.y >> 8) & 0xFF, ns = (U.y >> 16) & 0xFF;
+                const int n_kv = (sp + 1) * U.w / ns - sp * U.w / ns;
+                for (int j = 0; j < n_kv; ++j, ++kv_count) {
+                    const uint32_t nxt = kv_count + 1;
+                    if (!(ok = wait_bar(bar(C::kVFull + (int)(kv_count % NV)), (kv_count / NV) & 1, ctl))) break;
+                    if (j + 1 < n_kv && !(ok = wait_bar(bar(C::kKFull + (int)(nxt % NK)), (nxt / NK) & 1, ctl)))
+                        break;
+                    ptx::mbar_arrive(bar(C::kPFull + 0));
+                    // one arrival per phase: the next one only once this phase has completed
+                    if (!(ok = wait_bar(bar(C::kPFull + 0), p_phase, ctl))) break;
+                    p_phase ^= 1u;
+                }
+            }
+        }
+        __syncwarp();
     } else if (warp == kWarpMMA) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
@@ -274,25 +357,46 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             uint32_t kv_count = 0, unit_i = 0;
             uint32_t p_phase = 0;  // bit q: parity of the next P_q phase
             bool ok = true;
+            // Shared-memory descriptors are built once; a K-step inside a 128-byte swizzle atom, a chunk or
+            // a stage only moves the start address, i.e. adds (bytes >> 4) to the descriptor's low field
+            // (no carry: shared addresses are below 256 KiB).
+            const uint64_t desc_q0 = ptx::sdesc_sw128(sb + C::kOffQ, 16, 1024);
+            const uint64_t desc_k0 = ptx::sdesc_sw128(sb + C::kOffK, 16, 1024);
+            const uint64_t desc_v0 = ptx::sdesc_sw128(sb + C::kOffV, C::kChunkBytes, 1024);
             auto issue_qk = [&](int q, int s) {
                 const uint32_t d_tmem = tmem + (uint32_t)(q * 128);
+                const uint64_t da = desc_q0 + (uint64_t)((q * C::kQTileBytes) >> 4);
+                const uint64_t db = desc_k0 + (uint64_t)((s * C::kKVTileBytes) >> 4);
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
-                    const uint32_t a_addr =
-                        sb + C::kOffQ + q * C::kQTileBytes + (kk >> 2) * C::kChunkBytes + (kk & 3) * 32;
-                    const uint32_t b_addr =
-                        sb + C::kOffK + s * C::kKVTileBytes + (kk >> 2) * C::kChunkBytes + (kk & 3) * 32;
-                    ptx::mma_ss(d_tmem, ptx::sdesc_sw128(a_addr, 16, 1024), ptx::sdesc_sw128(b_addr, 16, 1024),
-                                idesc_qk, kk > 0 ? 1u : 0u);
+                    const uint64_t off = (uint64_t)((((kk >> 2) * C::kChunkBytes) + (kk & 3) * 32) >> 4);
+                    ptx::mma_ss(d_tmem, da + off, db + off, idesc_qk, kk > 0 ? 1u : 0u);
                 }
+            };
+            // the same, with a non-blocking test of (bar, parity) issued ahead of the last two MMAs
+            auto issue_qk_test = [&](int q, int s, uint32_t tbar, uint32_t parity) -> bool {
+                const uint32_t d_tmem = tmem + (uint32_t)(q * 128);
+                const uint64_t da = desc_q0 + (uint64_t)((q * C::kQTileBytes) >> 4);
+                const uint64_t db = desc_k0 + (uint64_t)((s * C::kKVTileBytes) >> 4);
+                constexpr int kSteps = D / 16;
+#pragma unroll
+                for (int kk = 0; kk < kSteps - 2; ++kk) {
+                    const uint64_t off = (uint64_t)((((kk >> 2) * C::kChunkBytes) + (kk & 3) * 32) >> 4);
+                    ptx::mma_ss(d_tmem, da + off, db + off, idesc_qk, kk > 0 ? 1u : 0u);
+                }
+                constexpr int k0 = kSteps - 2, k1 = kSteps - 1;
+                const uint64_t off0 = (uint64_t)((((k0 >> 2) * C::kChunkBytes) + (k0 & 3) * 32) >> 4);
+                const uint64_t off1 = (uint64_t)((((k1 >> 2) * C::kChunkBytes) + (k1 & 3) * 32) >> 4);
+                return ptx::mma_ss2_test(d_tmem, da + off0, db + off0, da + off1, db + off1, idesc_qk, 1u, tbar,
+                                         parity) != 0;
             };
             auto issue_pv = [&](int q, int s, bool accumulate) {
                 const uint32_t d_tmem = tmem + 256u + (uint32_t)(q * D);
+                const uint64_t db = desc_v0 + (uint64_t)((s * C::kKVTileBytes) >> 4);
 #pragma unroll
                 for (int kk = 0; kk < kBN / 16; ++kk) {
                     const uint32_t a_tmem = tmem + (uint32_t)(q * 128 + kk * 8);  // P: bf16 pairs over S_q
-                    const uint32_t b_addr = sb + C::kOffV + s * C::kKVTileBytes + kk * 16 * 128;
-                    ptx::mma_ts(d_tmem, a_tmem, ptx::sdesc_sw128(b_addr, C::kChunkBytes, 1024), idesc_pv,
+                    ptx::mma_ts(d_tmem, a_tmem, db + (uint64_t)((kk * 16 * 128) >> 4), idesc_pv,
                                 (accumulate || kk > 0) ? 1u : 0u);
                 }
             };
@@ -303,7 +407,6 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                 const int sp = (U.y >> 8) & 0xFF, ns = (U.y >> 16) & 0xFF;
                 const int n_kv = (sp + 1) * U.w / ns - sp * U.w / ns;  // KV tiles of this item
                 if (!(ok = wait_bar(bar(C::kQFull), unit_i & 1, ctl))) break;
-                ptx::tc_fence_after();
                 {
                     const int sk = (int)(kv_count % NK);
                     if (!(ok = wait_bar(bar(C::kKFull + sk), (kv_count / NK) & 1, ctl))) break;
@@ -314,55 +417,34 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                     ptx::mma_commit(bar(C::kSFull + 1));
                     ptx::mma_commit(bar(C::kKEmpty + sk));
                 }
+                // P_q waits: a test for the next P rides on the last MMAs of the S GEMM before it; the
+                // blocking wait runs only when that test found the phase still open.
+                bool p_ready[kNQ] = {false, false};
                 for (int j = 0; j < n_kv && ok; ++j) {
                     const uint32_t cur = kv_count + j, nxt = cur + 1;
                     const int sv = (int)(cur % NV), sk1 = (int)(nxt % NK);
                     const bool more = j + 1 < n_kv;
-                    if (!(ok = wait_bar(bar(C::kVFull + sv), (cur / NV) & 1, ctl))) break;
-                    ptx::tc_fence_after();
-                    if constexpr (kPVFirst) {
-                        // PV_0(j), PV_1(j), S_0(j+1), S_1(j+1): no two adjacent MMAs touch the same TMEM columns
+                    // PV_0(j), S_0(j+1), PV_1(j), S_1(j+1).  V(j) and K(j+1) are not waited for here: P_0(j)
+                    // completes only after the stage warp has seen both land.
 #pragma unroll
-                        for (int q = 0; q < kNQ; ++q) {
-                            if (!(ok = wait_bar(bar(C::kPFull + q), (p_phase >> q) & 1u, ctl))) break;
-                            p_phase ^= 1u << q;
-                            ptx::tc_fence_after();
-                            issue_pv(q, sv, j > 0);
-                            if (!more) ptx::mma_commit(bar(C::kOFinal + q));
+                    for (int q = 0; q < kNQ; ++q) {
+                        if (!p_ready[q] && !(ok = wait_bar(bar(C::kPFull + q), (p_phase >> q) & 1u, ctl))) break;
+                        p_ready[q] = false;  // consumed
+                        p_phase ^= 1u << q;
+                        ptx::tc_fence_after();
+                        issue_pv(q, sv, j > 0);
+                        if (!more) {
+                            ptx::mma_commit(bar(C::kOFinal + q));
+                            continue;
                         }
-                        if (!ok) break;
-                        ptx::mma_commit(bar(C::kVEmpty + sv));
-                        if (more) {
-                            if (!(ok = wait_bar(bar(C::kKFull + sk1), (nxt / NK) & 1, ctl))) break;
-                            ptx::tc_fence_after();
-                            issue_qk(0, sk1);
-                            ptx::mma_commit(bar(C::kSFull + 0));
-                            issue_qk(1, sk1);
-                            ptx::mma_commit(bar(C::kSFull + 1));
-                            ptx::mma_commit(bar(C::kKEmpty + sk1));
-                        }
-                    } else {
-                        // PV_0(j), S_0(j+1), PV_1(j), S_1(j+1): one Q tile's MMAs overlap the other's softmax
-#pragma unroll
-                        for (int q = 0; q < kNQ; ++q) {
-                            if (!(ok = wait_bar(bar(C::kPFull + q), (p_phase >> q) & 1u, ctl))) break;
-                            p_phase ^= 1u << q;
-                            ptx::tc_fence_after();
-                            issue_pv(q, sv, j > 0);
-                            if (!more) ptx::mma_commit(bar(C::kOFinal + q));
-                            if (more) {
-                                if (q == 0) {
-                                    if (!(ok = wait_bar(bar(C::kKFull + sk1), (nxt / NK) & 1, ctl))) break;
-                                    ptx::tc_fence_after();
-                                }
-                                issue_qk(q, sk1);
-                                ptx::mma_commit(bar(C::kSFull + q));
-                                if (q == kNQ - 1) ptx::mma_commit(bar(C::kKEmpty + sk1));
-                            }
-                        }
-                        if (!ok) break;
-                        ptx::mma_commit(bar(C::kVEmpty + sv));
+                        // test the P the next PV needs: P_1(j) after S_0(j+1), P_0(j+1) after S_1(j+1)
+                        const int qn = (q + 1) % kNQ;
+                        p_ready[qn] = issue_qk_test(q, sk1, bar(C::kPFull + qn), (p_phase >> qn) & 1u);
+                        ptx::mma_commit(bar(C::kSFull + q));
+                        if (q == kNQ - 1) ptx::mma_commit(bar(C::kKEmpty + sk1));
                     }
+                    if (!ok) break;
+                    ptx::mma_commit(bar(C::kVEmpty + sv));
                 }
                 if (!ok) break;
                 ptx::mma_commit(bar(C::kQEmpty));
@@ -373,11 +455,25 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                 ptx::mma_commit(bar(C::kDrain));
                 drain_bar(bar(C::kDrain), 0);
             }
+            // TMEM is freed once every softmax thread has finished its last TMEM access (bounded like every
+            // other wait; the columns must be released in any case, or the next kernel on this SM could not
+            // allocate them)
+            {
+                const long long t0 = clock64();
+                while (!ptx::mbar_try_wait_sleep(bar(C::kDone), 0, 200000u))
+                    if (clock64() - t0 > kWaitLimitCycles) { atomicCAS(a.err, 0, RR_ERR_TIMEOUT); break; }
+            }
         }
         __syncwarp();
-    } else {
-        // ------------------------------------------------------------ softmax warpgroups
-        const int q = warp >> 2;              // Q tile of this warpgroup
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem, 512);
+    }
+    return;
+    }
+    // ================================================================ softmax warpgroups (warps 0-7)
+    ptx::setmaxnreg_inc<kRegsSoftmax>();
+    {
+        const int q = warp >> 2;                // Q tile of this warpgroup
         const int r = threadIdx.x & (kBM - 1);  // row == TMEM lane
         const uint32_t lane_bits = (uint32_t)((warp & 3) * 32) << 16;
         const uint32_t t_s = tmem + lane_bits + (uint32_t)(q * 128);
@@ -393,8 +489,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             const int kb = sp * U.w / ns, ke = (sp + 1) * U.w / ns;  // this item's KV tiles
             const int P = a.prefix[b], agent_len = P + a.suffix[b];
             const int tq0 = u * unit_tokens + q * a.tq;  // first suffix token of this Q tile
-            const int tok = tq0 + r / a.G;
-            const int row_limit = min(P + tok, agent_len - 1);     // last key this row may see
+            const int row_limit = min(P + tq0 + r / a.G, agent_len - 1);     // last key this row may see
             const int mask_from = (min(P + tq0, agent_len - 1) + 1) / kBN;  // earlier tiles: no masking
             float m_run = -INFINITY, l_run = 0.f;
             for (int j = kb; j < ke; ++j) {
@@ -450,16 +545,22 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                     l_run *= f;
                     m_run = mxs;
                 }
-                const float neg = m_run == -INFINITY ? 0.f : -m_run;  // a fully masked row stays at p = 0
-                // p = 2^(s * scale * log2e - m): packed FMA, ex2, packed accumulation over 8 chains
+                const float neg = m_run == -INFINITY ? 0.f : -m_run;  // a fully masked row keeps p = 0
+                // p = 2^(s * scale * log2e - m): packed FMA, ex2, packed accumulation over 8 chains; the
+                // first half of P goes to TMEM while the second is computed
                 float la[4] = {0.f, 0.f, 0.f, 0.f}, lb[4] = {0.f, 0.f, 0.f, 0.f};
                 uint32_t pk[kBN / 2];
 #pragma unroll
                 for (int c = 0; c < kBN; c += 2) {
-                    float x0, x1;
+                    float x0, x1, p0, p1;
                     ptx::fma2(x0, x1, sv[c], sv[c + 1], sl2, sl2, neg, neg);
-                    const float p0 = ptx::ex2_approx(x0);
-                    const float p1 = ptx::ex2_approx(x1);
+                    if (kEmuPairStride > 0 && (c >> 1) % (kEmuPairStride > 0 ? kEmuPairStride : 1) ==
+                                                  (kEmuPairStride > 0 ? kEmuPairStride - 1 : 0)) {
+                        exp2_poly2(p0, p1, x0, x1);
+                    } else {
+                        p0 = ptx::ex2_approx(x0);
+                        p1 = ptx::ex2_approx(x1);
+                    }
                     const int k = (c >> 1) & 3;
                     ptx::add2(la[k], lb[k], la[k], lb[k], p0, p1);
                     pk[c >> 1] = ptx::pack_bf16x2(p0, p1);
@@ -512,10 +613,10 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                 continue;
             }
             const float inv_l = 1.0f / l_run;
-            const int tok_e = u * unit_tokens + q * a.tq + r / a.G;  // recomputed: keeps the tile loop lean
-            const bool valid = tok_e < a.suffix[b];
+            const int tok = tq0 + r / a.G;
+            const bool valid = tok < a.suffix[b];
             __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(a.out) +
-                                 ((long long)(a.cu[b] + tok_e) * a.Hq + g * a.G + r % a.G) * D;
+                                 ((long long)(a.cu[b] + tok) * a.Hq + g * a.G + r % a.G) * D;
 #pragma unroll
             for (int c = 0; c < D; c += 32) {
                 uint32_t o[32];
@@ -533,16 +634,11 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             }
         }
     }
-
     ptx::tc_fence_before();
-    __syncthreads();
-    if (warp == kWarpMMA) {
-        ptx::tc_fence_after();
-        ptx::tmem_dealloc(tmem, 512);
-    }
+    ptx::mbar_arrive(bar(C::kDone));
 }
 
-template <int D, int NK, int NV, bool kPVFirst>
+template <int D, int NK, int NV>
 cudaError_t launch_cfg(const AttnArgs& a, int grid, cudaStream_t st) {
     using C = Cfg<D, NK, NV>;
     static bool attr_done[64] = {};
@@ -551,26 +647,26 @@ cudaError_t launch_cfg(const AttnArgs& a, int grid, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     if (!attr_done[dev]) {
-        e = cudaFuncSetAttribute(extend_attn_kernel<D, NK, NV, kPVFirst>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(extend_attn_kernel<D, NK, NV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  C::kSmemBytes);
         if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
-    extend_attn_kernel<D, NK, NV, kPVFirst><<<grid, kThreads, C::kSmemBytes, st>>>(a);
+    extend_attn_kernel<D, NK, NV><<<grid, kThreads, C::kSmemBytes, st>>>(a);
     return cudaGetLastError();
 }
 
 }  // namespace
 
 size_t extend_attention_smem_bytes(int head_dim) {
-    if (head_dim == 128) return Cfg<128, 2, 2>::kSmemBytes;
+    if (head_dim == 128) return Cfg<128, 2, 3>::kSmemBytes;
     if (head_dim == 64) return Cfg<64, 4, 4>::kSmemBytes;
     return 0;
 }
 
 cudaError_t launch_extend_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st) {
-    if (head_dim == 128) return launch_cfg<128, 2, 2, false>(a, grid, st);
-    if (head_dim == 64) return launch_cfg<64, 4, 4, false>(a, grid, st);
+    if (head_dim == 128) return launch_cfg<128, 2, 3>(a, grid, st);
+    if (head_dim == 64) return launch_cfg<64, 4, 4>(a, grid, st);
     return cudaErrorInvalidValue;
 }
 

@@ -145,6 +145,28 @@ __device__ __forceinline__ void mma_ss(uint32_t d_tmem, uint64_t a_desc, uint64_
         : "memory");
 }
 
+// Two SS MMAs (the second always accumulates) with a non-blocking test of an mbarrier phase in front
+// of them, in one asm block: the test's latency overlaps the MMA issue, and its result is returned
+// (1: the phase with the given parity has completed) without stalling the MMAs behind it.
+__device__ __forceinline__ uint32_t mma_ss2_test(uint32_t d_tmem, uint64_t a0, uint64_t b0, uint64_t a1,
+                                                 uint64_t b1, uint32_t idesc, uint32_t accumulate0,
+                                                 uint32_t bar, uint32_t parity) {
+    uint32_t ready;
+    asm volatile(
+        "{\n\t.reg .pred pr, pa;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 pr, [%8], %9;\n\t"
+        "setp.ne.b32 pa, %7, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%1], %2, %3, %6, pa;\n\t"
+        "setp.ne.b32 pa, %10, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%1], %4, %5, %6, pa;\n\t"
+        "selp.u32 %0, 1, 0, pr;\n\t}"
+        : "=r"(ready)
+        : "r"(d_tmem), "l"(a0), "l"(b0), "l"(a1), "l"(b1), "r"(idesc), "r"(accumulate0), "r"(bar), "r"(parity),
+          "r"(1u)
+        : "memory");
+    return ready;
+}
+
 // D[tmem] (+)= A[tmem] * B[smem]
 __device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
                                        uint32_t accumulate) {
