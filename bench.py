@@ -275,6 +275,59 @@ def per_agent_latency(rr, wl, g, dev, st, reps=5):
             "p50_ms": float(np.percentile(t, 50)), "mean_ms": float(t.mean()), "sum_ms": float(t.sum())}
 
 
+def decode_bytes(wl) -> float:
+    """Algorithmic bytes of one decode call: each agent's K and V once per KV head, q in, out out, the page
+    table entries and lengths read."""
+    kv_tok = float((wl.prefix_lens.astype(np.int64) + 1).sum())
+    pages = float(sum(-(-(int(p) + 1) // wl.ps) for p in wl.prefix_lens))
+    return kv_tok * wl.Hkv * wl.D * 2 * 2 + 2.0 * wl.B * wl.Hq * wl.D * 2 + pages * 4 + wl.B * 4
+
+
+def decode_leg(args, rr, synth, dev, st, peaks, rank):
+    """Decode attention on a decode batch (one new token per agent), device-timed per call."""
+    import torch
+    free = torch.cuda.mem_get_info(dev)[0]
+    wl = synth.decode_config(args.decode_config, seed=rank,
+                             free_hbm_bytes=free if args.decode_config == "c4_decode" else None)
+    if args.decode_agents:
+        n = args.decode_agents
+        wl = synth.custom(f"{args.decode_config}[:{n}]", n, wl.Hq, wl.Hkv, wl.D, wl.prefix_lens[:n],
+                          wl.suffix_lens[:n], ps=wl.ps, shared_len=wl.shared_len, seed=wl.seed)
+    g = synth.gpu_tensors(wl, dev)
+    rr.kv_append(g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                 g["suffix_lens"])
+    kv_lens = (g["prefix_lens"] + 1).to(torch.int32)
+    out = torch.empty_like(g["q"])
+    for _ in range(max(3, args.warmup)):
+        rr.decode_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"], kv_lens, out=out)
+    torch.cuda.synchronize(dev)
+    if rr.device_error():
+        raise RuntimeError("device error in the decode warm-up")
+    n = max(args.steps, 10)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+    for e0, e1 in ev:
+        e0.record(st)
+        rr.decode_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"], kv_lens, out=out)
+        e1.record(st)
+    torch.cuda.synchronize(dev)
+    if rr.device_error():
+        raise RuntimeError("device error in the decode timed region")
+    ms = statistics.mean(e0.elapsed_time(e1) for e0, e1 in ev)
+    nbytes = decode_bytes(wl)
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    res = {"workload": wl.name, "B": wl.B, "Hq": wl.Hq, "Hkv": wl.Hkv, "D": wl.D,
+           "kv_tokens": int((wl.prefix_lens.astype(np.int64) + 1).sum()), "calls": n, "ms_per_call": ms,
+           "tokens_per_s": wl.B / (ms * 1e-3),
+           "roofline": {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm"], "unit": "GB/s",
+                        "frac": gbs / peaks["hbm"], "traffic": None, "algorithmic_bytes": nbytes,
+                        "kernel": f"decode_attn_kernel<{wl.D},{3 if wl.D == 128 else 6},{wl.G}>",
+                        "peak_kind": f"{peaks['src']} HBM copy bandwidth"},
+           "l2": f"K/V working set {nbytes / 1e9:.1f} GB > 129 MB"}
+    del g, out, kv_lens
+    torch.cuda.empty_cache()
+    return res
+
+
 def run_ours(args, world, rank, local):
     import torch
     import synth
@@ -381,6 +434,11 @@ def run_ours(args, world, rank, local):
     per_agent = None
     if args.per_agent:
         per_agent = per_agent_latency(rr, wl, g, dev, st)
+    decode = None
+    if not args.no_decode:
+        g.clear()
+        torch.cuda.empty_cache()
+        decode = decode_leg(args, rr, synth, dev, st, peaks, rank)
 
     achieved = F / (attn_ms * 1e-3) / 1e12
     src_hash = kernel_source_hash()
@@ -415,6 +473,8 @@ def run_ours(args, world, rank, local):
     }
     if per_agent is not None:
         line["per_agent_extend"] = per_agent
+    if decode is not None:
+        line["decode"] = decode
     if rank == 0 and not args.no_cpu_baseline:
         f, t, rows, threads = cpu_oracle_sample(wl, args.baseline_flops, seed=7)
         line["cpu_baseline"] = {"value": f / t / 1e12, "unit": "TFLOP/s", "cores": threads, "kind": "oracle",
@@ -438,6 +498,9 @@ def main():
     ap.add_argument("--agents", type=int, default=0, help="only the first N agents (small profiling case)")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
     ap.add_argument("--per-agent", action="store_true", help="also time each agent's extend step alone")
+    ap.add_argument("--decode-config", default="c2_decode", help="decode batch of the decode leg")
+    ap.add_argument("--no-decode", action="store_true", help="skip the decode-attention leg")
+    ap.add_argument("--decode-agents", type=int, default=0, help="only the first N agents of the decode batch")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

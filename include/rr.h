@@ -112,6 +112,34 @@ int rr_extend_attention(const void* q, const void* k_pool, const void* v_pool, c
                         float softmax_scale, cudaStream_t stream);
 
 /*
+ * rr_decode_attention -- decode attention over the same paged pool: the
+ * extend attention above for a suffix of exactly one token per agent, the
+ * step that follows an extend in an agent's turn (Sec. 2: an agent's request
+ * reuses the cached KV and computes only what is new).
+ *
+ * q [B][Hq][D] bf16: the one new query token of each agent (row b is agent b).
+ * kv_lens [B] int32 (device): L_b >= 1 keys of agent b in the pool, the new
+ * token's own K/V included (append it first with rr_kv_append, prefix_lens =
+ * L_b - 1, suffix_lens = 1).  out [B][Hq][D] bf16.  dims: total_tokens must
+ * equal batch; the other fields as for rr_extend_attention.
+ *     out[b, h, :] = sum_j softmax_j(scale * <q[b, h, :], K_j>) V_j,  j < L_b
+ * with K_j, V_j position j of agent b, KV head h / G, through page_table.
+ *
+ * Same accuracy, determinism and page-placement independence as
+ * rr_extend_attention; a kernel built for one query row per KV head (the
+ * tensor cores take the keys as rows), bound by HBM bandwidth.  Batches with
+ * few (agent, KV head) pairs split each agent's keys over several CTAs and
+ * merge the pieces, as rr_extend_attention does.  Errors: RR_ERR_INVALID_ARG
+ * (nulls, misalignment, total_tokens != batch), RR_ERR_UNSUPPORTED as for
+ * rr_extend_attention; on the device a length L_b < 1 or L_b > max_pages *
+ * page_size records RR_ERR_LENS and a page id outside the pool RR_ERR_OOB.
+ * Allocates only the library's cached per-device workspace.
+ */
+int rr_decode_attention(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
+                        const int32_t* kv_lens, void* out, const rr_dims* dims, float softmax_scale,
+                        cudaStream_t stream);
+
+/*
  * rr_extend_attention_noalloc -- rr_extend_attention for callers that cannot
  * allocate device memory.  The paper has no counterpart; this is a deployment
  * convenience of this library.

@@ -109,6 +109,19 @@ def extend_attention(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, sc
     return (out, lse, wsum) if with_stats else out
 
 
+def decode_attention(q, k_pool, v_pool, page_table, kv_lens, scale=None, nthreads=0, with_stats=False):
+    """Decode attention: out [B, Hq, D] float64 -- the extend definition (Sec. 2) for a suffix of one token
+    per agent.  Row b is agent b's new token, at position kv_lens[b] - 1; it sees all kv_lens[b] keys.
+
+    No arithmetic of its own: the lengths are restated (prefix = L - 1, suffix = 1) and the extend
+    oracle computes the plain definition."""
+    L = _c(kv_lens, np.int32)
+    if (L < 1).any():
+        raise OracleError("decode_attention: every agent needs at least its own key")
+    return extend_attention(q, k_pool, v_pool, page_table, L - 1, np.ones_like(L), scale=scale, nthreads=nthreads,
+                            with_stats=with_stats)
+
+
 def attention_rows(q_rows, positions, K, V, scale, nthreads=0, with_stats=False):
     """Selected rows of one agent / one KV group over its logical K, V ([n_keys, D] bf16 bits).
 

@@ -7,6 +7,11 @@ suffix):
     kv_append(k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens)
     out = extend_attention(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens)
 
+and the step after it, one new token per agent:
+
+    kv_append(k_tok, v_tok, k_pool, v_pool, page_table, kv_lens - 1, ones)
+    out = decode_attention(q_tok, k_pool, v_pool, page_table, kv_lens)
+
 This module only marshals torch tensors into the C ABI of include/rr.h; every
 step of the computation runs in the CUDA kernels of librr.so.  There is no
 fallback: if the library is missing or a call fails, an exception is raised.
@@ -30,8 +35,8 @@ RR_ERR_LENS = 6
 RR_ERR_OVERLAP = 7
 
 # Every symbol include/rr.h declares.
-EXPORTS = ("rr_kv_append", "rr_extend_attention", "rr_validate_page_table", "rr_get_device_error",
-           "rr_last_error", "rr_version", "rr_shutdown", "rr_extend_attention_noalloc")
+EXPORTS = ("rr_kv_append", "rr_extend_attention", "rr_decode_attention", "rr_validate_page_table",
+           "rr_get_device_error", "rr_last_error", "rr_version", "rr_shutdown", "rr_extend_attention_noalloc")
 
 
 class RRError(RuntimeError):
@@ -68,6 +73,8 @@ def lib():
         L.rr_kv_append.argtypes = [vp, vp, vp, vp, vp, vp, vp, dp, vp]
         L.rr_extend_attention.restype = ctypes.c_int
         L.rr_extend_attention.argtypes = [vp, vp, vp, vp, vp, vp, vp, dp, ctypes.c_float, vp]
+        L.rr_decode_attention.restype = ctypes.c_int
+        L.rr_decode_attention.argtypes = [vp, vp, vp, vp, vp, vp, dp, ctypes.c_float, vp]
         L.rr_validate_page_table.restype = ctypes.c_int
         L.rr_validate_page_table.argtypes = [vp, vp, vp, dp]
         L.rr_get_device_error.restype = ctypes.c_int
@@ -162,6 +169,35 @@ def extend_attention(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, ou
     _check(lib().rr_extend_attention(q.data_ptr(), k_pool.data_ptr(), v_pool.data_ptr(), page_table.data_ptr(),
                                      prefix_lens.data_ptr(), suffix_lens.data_ptr(), out.data_ptr(),
                                      ctypes.byref(dims), float(softmax_scale), _stream_ptr(stream, q.device)))
+    return out
+
+
+def decode_attention(q, k_pool, v_pool, page_table, kv_lens, out=None, softmax_scale: float = 0.0, stream=None):
+    """Decode attention: the one new query token of each agent over its kv_lens[b] keys (rr_decode_attention).
+
+    q: [B, Hq, D] bf16; kv_lens: [B] int32, the new token's K/V already appended."""
+    import torch
+    _need(q, "q", torch.bfloat16, 3)
+    _need(k_pool, "k_pool", torch.bfloat16, 4)
+    _need(v_pool, "v_pool", torch.bfloat16, 4)
+    _need(page_table, "page_table", torch.int32, 2)
+    _need(kv_lens, "kv_lens", torch.int32, 1)
+    B, Hq, D = q.shape
+    num_pages, ps, Hkv, D2 = k_pool.shape
+    if v_pool.shape != k_pool.shape or D2 != D:
+        raise ValueError("q / pool shapes disagree")
+    if kv_lens.shape[0] != B or page_table.shape[0] != B:
+        raise ValueError("q / kv_lens / page_table batch sizes disagree")
+    if out is None:
+        out = torch.empty_like(q)
+    else:
+        _need(out, "out", torch.bfloat16, 3)
+        if out.shape != q.shape:
+            raise ValueError("out must have q's shape")
+    dims = make_dims(B, Hq, Hkv, D, ps, page_table.shape[1], num_pages, B)
+    _check(lib().rr_decode_attention(q.data_ptr(), k_pool.data_ptr(), v_pool.data_ptr(), page_table.data_ptr(),
+                                     kv_lens.data_ptr(), out.data_ptr(), ctypes.byref(dims), float(softmax_scale),
+                                     _stream_ptr(stream, q.device)))
     return out
 
 

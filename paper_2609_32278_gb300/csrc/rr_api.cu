@@ -46,11 +46,13 @@ size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 // Workspace layout: [n_units, lens_ok, n_split][cu: B+1][unit_off: B+1][items: max_items x int4]
 // [item_slot: max_items][split units: max_split x int4][part_ml: slots x 256 float2][part_o: slots x 256 x D]
+// [decode only: prefix B][suffix B]
 struct Layout {
-    size_t off_cu, off_unit_off, off_units, off_slot, off_split, off_ml, off_o, total;
+    size_t off_cu, off_unit_off, off_units, off_slot, off_split, off_ml, off_o, off_lens, total;
 };
 
-Layout layout_for(int64_t B, int64_t max_items, int64_t max_split = 0, int64_t slots = 0, int64_t D = 0) {
+Layout layout_for(int64_t B, int64_t max_items, int64_t max_split = 0, int64_t slots = 0, int64_t D = 0,
+                  bool lens = false) {
     Layout L;
     L.off_cu = 256;
     L.off_unit_off = L.off_cu + align256((size_t)(B + 1) * 4);
@@ -59,7 +61,8 @@ Layout layout_for(int64_t B, int64_t max_items, int64_t max_split = 0, int64_t s
     L.off_split = L.off_slot + align256((size_t)max_items * 4);
     L.off_ml = L.off_split + align256((size_t)max_split * 16);
     L.off_o = L.off_ml + align256((size_t)slots * rr::kNQ * rr::kBM * 8);
-    L.total = L.off_o + align256((size_t)slots * rr::kNQ * rr::kBM * (size_t)D * 4);
+    L.off_lens = L.off_o + align256((size_t)slots * rr::kNQ * rr::kBM * (size_t)D * 4);
+    L.total = L.off_lens + (lens ? 2 * align256((size_t)B * 4) : 0);  // decode: prefix, suffix arrays
     return L;
 }
 
@@ -169,6 +172,143 @@ int encode_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64
 
 }  // namespace
 
+namespace {
+
+// Extend attention, or decode attention (decode = true: kv_lens in place of the prefix / suffix lengths,
+// one query token per agent, the decode kernel in place of the extend kernel).
+int attention_impl(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
+                   const int32_t* prefix_lens, const int32_t* suffix_lens, const int32_t* kv_lens, void* out,
+                   const rr_dims* dims, float softmax_scale, cudaStream_t stream, bool decode) {
+    g_msg[0] = 0;
+    int rc = check_dims(dims, true);
+    if (rc) return rc;
+    if (dims->total_tokens == 0 && dims->batch == 0) return RR_OK;
+    if (decode) {
+        if (!page_table || !kv_lens) return fail(RR_ERR_INVALID_ARG, "null kv_lens or page table");
+        if (dims->total_tokens != dims->batch)
+            return fail(RR_ERR_INVALID_ARG, "decode takes one query token per agent: total_tokens (%lld) != batch (%d)",
+                        (long long)dims->total_tokens, dims->batch);
+        if (!aligned4(kv_lens)) return fail(RR_ERR_INVALID_ARG, "int32 arrays must be 4-byte aligned");
+    } else if (!page_table || !prefix_lens || !suffix_lens) {
+        return fail(RR_ERR_INVALID_ARG, "null lens or page table");
+    }
+    if (dims->total_tokens > 0 && (!q || !k_pool || !v_pool || !out))
+        return fail(RR_ERR_INVALID_ARG, "null q/pool/out pointer");
+    if (!aligned16(q) || !aligned16(k_pool) || !aligned16(v_pool) || !aligned16(out))
+        return fail(RR_ERR_INVALID_ARG, "q, pools and out must be 16-byte aligned");
+    if (!aligned4(page_table) || (!decode && (!aligned4(prefix_lens) || !aligned4(suffix_lens))))
+        return fail(RR_ERR_INVALID_ARG, "int32 arrays must be 4-byte aligned");
+    if (dims->total_tokens > 0 && dims->num_pages == 0) return fail(RR_ERR_INVALID_ARG, "empty pool");
+    const int Hq = dims->num_q_heads, Hkv = dims->num_kv_heads, D = dims->head_dim, ps = dims->page_size;
+    const int G = Hq / Hkv;
+    const int tq = rr::kBM / G;
+    const int unit_tokens = rr::kNQ * tq;
+    const int64_t T = dims->total_tokens, B = dims->batch;
+    const int64_t max_units = (int64_t)Hkv * (T / unit_tokens + B + 1);
+    if (max_units >= (1ll << 31)) return fail(RR_ERR_UNSUPPORTED, "too many work units");
+
+    Device* d = nullptr;
+    if ((rc = current_device(&d, nullptr))) return rc;
+    if ((rc = get_encoder())) return rc;
+    // Split-K is possible only when the batch may have fewer than two waves of units; the batch has at
+    // least Hkv * T / unit_tokens units, so larger batches never split and need no partial buffers.
+    const int grid_sm = d->sm_count;
+    const bool may_split = (int64_t)Hkv * (T / unit_tokens) < 2ll * grid_sm;
+    const int64_t max_split = may_split ? 2ll * grid_sm : 0;
+    const int64_t slots = may_split ? 4ll * grid_sm : 0;
+    const int64_t max_items = std::max<int64_t>(max_units, slots);
+    const Layout L = layout_for(B, max_items, max_split, slots, D, decode);
+    if ((rc = ensure_ws(*d, L.total))) return rc;
+    uint8_t* ws = static_cast<uint8_t*>(d->ws);
+    cudaError_t e = cudaSuccess;
+    if (decode) {
+        int32_t* pre = reinterpret_cast<int32_t*>(ws + L.off_lens);
+        int32_t* suf = reinterpret_cast<int32_t*>(ws + L.off_lens + align256((size_t)B * 4));
+        e = rr::launch_decode_lens(kv_lens, pre, suf, (int32_t)B, d->err, stream);
+        if (e != cudaSuccess) return cuda_fail(e, "decode lengths kernel launch");
+        prefix_lens = pre;
+        suffix_lens = suf;
+    }
+
+    rr::SchedArgs s{};
+    s.prefix = prefix_lens;
+    s.suffix = suffix_lens;
+    s.B = (int32_t)B;
+    s.Hkv = Hkv;
+    s.unit_tokens = unit_tokens;
+    s.T = T;
+    s.max_pages = dims->max_pages;
+    s.ps = ps;
+    s.max_units = max_units;
+    s.build_units = 1;
+    s.cu = reinterpret_cast<int32_t*>(ws + L.off_cu);
+    s.unit_off = reinterpret_cast<int32_t*>(ws + L.off_unit_off);
+    s.units = reinterpret_cast<int4*>(ws + L.off_units);
+    s.item_slot = reinterpret_cast<int32_t*>(ws + L.off_slot);
+    s.split_units = reinterpret_cast<int4*>(ws + L.off_split);
+    s.n_split = reinterpret_cast<int32_t*>(ws) + 2;
+    s.split_grid = may_split ? grid_sm : 0;
+    s.n_units = reinterpret_cast<int32_t*>(ws);
+    s.lens_ok = reinterpret_cast<int32_t*>(ws) + 1;
+    s.err = d->err;
+    e = rr::launch_sched(s, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "schedule kernel launch");
+    if (T == 0) return RR_OK;
+
+    rr::AttnArgs a;
+    memset(&a, 0, sizeof a);
+    // q [T][Hq][D]: a box is one 64-column chunk of G heads x (128/G tokens, or the one token of decode)
+    if ((rc = encode_3d(&a.tm_q, q, (uint64_t)D, (uint64_t)Hq, (uint64_t)T, (uint64_t)D * 2, (uint64_t)Hq * D * 2, 64,
+                        (uint32_t)G, decode ? 1u : (uint32_t)tq)))
+        return rc;
+    const uint64_t rows = (uint64_t)dims->num_pages * (uint64_t)ps;
+    if ((rc = encode_2d(&a.tm_k, k_pool, (uint64_t)Hkv * D, rows, (uint64_t)Hkv * D * 2, 64, (uint32_t)ps))) return rc;
+    if ((rc = encode_2d(&a.tm_v, v_pool, (uint64_t)Hkv * D, rows, (uint64_t)Hkv * D * 2, 64, (uint32_t)ps))) return rc;
+    a.page_table = page_table;
+    a.prefix = prefix_lens;
+    a.suffix = suffix_lens;
+    a.cu = s.cu;
+    a.units = s.units;
+    a.n_units = s.n_units;
+    a.item_slot = s.item_slot;
+    a.part_o = reinterpret_cast<float*>(ws + L.off_o);
+    a.part_ml = reinterpret_cast<float2*>(ws + L.off_ml);
+    a.err = d->err;
+    a.out = out;
+    a.num_pages = dims->num_pages;
+    a.Hq = Hq;
+    a.G = G;
+    a.ps = ps;
+    a.max_pages = dims->max_pages;
+    a.tq = tq;
+    a.oob_row = (int32_t)rows;
+    const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)D);
+    a.scale_log2 = scale * 1.4426950408889634f;
+    const int64_t grid = std::min<int64_t>((int64_t)d->sm_count, max_items);
+    e = decode ? rr::launch_decode_attention(a, D, (int)std::max<int64_t>(grid, 1), stream)
+               : rr::launch_extend_attention(a, D, (int)std::max<int64_t>(grid, 1), stream);
+    if (e != cudaSuccess) return cuda_fail(e, decode ? "decode attention kernel launch" : "extend attention kernel launch");
+    if (may_split) {
+        rr::CombineArgs c;
+        c.split_units = s.split_units;
+        c.n_split = s.n_split;
+        c.part_o = a.part_o;
+        c.part_ml = a.part_ml;
+        c.suffix = suffix_lens;
+        c.cu = s.cu;
+        c.out = out;
+        c.Hq = Hq;
+        c.G = G;
+        c.D = D;
+        c.tq = tq;
+        e = rr::launch_combine(c, (int)max_split, stream);
+        if (e != cudaSuccess) return cuda_fail(e, "split-K combine kernel launch");
+    }
+    return RR_OK;
+}
+
+}  // namespace
+
 extern "C" {
 
 const char* rr_version(void) { return "rr-extend 0.1 (sm_103a)"; }
@@ -243,113 +383,15 @@ int rr_kv_append(const void* k_new, const void* v_new, void* k_pool, void* v_poo
 int rr_extend_attention(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
                         const int32_t* prefix_lens, const int32_t* suffix_lens, void* out, const rr_dims* dims,
                         float softmax_scale, cudaStream_t stream) {
-    g_msg[0] = 0;
-    int rc = check_dims(dims, true);
-    if (rc) return rc;
-    if (dims->total_tokens == 0 && dims->batch == 0) return RR_OK;
-    if (!page_table || !prefix_lens || !suffix_lens) return fail(RR_ERR_INVALID_ARG, "null lens or page table");
-    if (dims->total_tokens > 0 && (!q || !k_pool || !v_pool || !out))
-        return fail(RR_ERR_INVALID_ARG, "null q/pool/out pointer");
-    if (!aligned16(q) || !aligned16(k_pool) || !aligned16(v_pool) || !aligned16(out))
-        return fail(RR_ERR_INVALID_ARG, "q, pools and out must be 16-byte aligned");
-    if (!aligned4(page_table) || !aligned4(prefix_lens) || !aligned4(suffix_lens))
-        return fail(RR_ERR_INVALID_ARG, "int32 arrays must be 4-byte aligned");
-    if (dims->total_tokens > 0 && dims->num_pages == 0) return fail(RR_ERR_INVALID_ARG, "empty pool");
-    const int Hq = dims->num_q_heads, Hkv = dims->num_kv_heads, D = dims->head_dim, ps = dims->page_size;
-    const int G = Hq / Hkv;
-    const int tq = rr::kBM / G;
-    const int unit_tokens = rr::kNQ * tq;
-    const int64_t T = dims->total_tokens, B = dims->batch;
-    const int64_t max_units = (int64_t)Hkv * (T / unit_tokens + B + 1);
-    if (max_units >= (1ll << 31)) return fail(RR_ERR_UNSUPPORTED, "too many work units");
+    return attention_impl(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, nullptr, out, dims, softmax_scale,
+                          stream, false);
+}
 
-    Device* d = nullptr;
-    if ((rc = current_device(&d, nullptr))) return rc;
-    if ((rc = get_encoder())) return rc;
-    // Split-K is possible only when the batch may have fewer than two waves of units; the batch has at
-    // least Hkv * T / unit_tokens units, so larger batches never split and need no partial buffers.
-    const int grid_sm = d->sm_count;
-    const bool may_split = (int64_t)Hkv * (T / unit_tokens) < 2ll * grid_sm;
-    const int64_t max_split = may_split ? 2ll * grid_sm : 0;
-    const int64_t slots = may_split ? 4ll * grid_sm : 0;
-    const int64_t max_items = std::max<int64_t>(max_units, slots);
-    const Layout L = layout_for(B, max_items, max_split, slots, D);
-    if ((rc = ensure_ws(*d, L.total))) return rc;
-    uint8_t* ws = static_cast<uint8_t*>(d->ws);
-
-    rr::SchedArgs s{};
-    s.prefix = prefix_lens;
-    s.suffix = suffix_lens;
-    s.B = (int32_t)B;
-    s.Hkv = Hkv;
-    s.unit_tokens = unit_tokens;
-    s.T = T;
-    s.max_pages = dims->max_pages;
-    s.ps = ps;
-    s.max_units = max_units;
-    s.build_units = 1;
-    s.cu = reinterpret_cast<int32_t*>(ws + L.off_cu);
-    s.unit_off = reinterpret_cast<int32_t*>(ws + L.off_unit_off);
-    s.units = reinterpret_cast<int4*>(ws + L.off_units);
-    s.item_slot = reinterpret_cast<int32_t*>(ws + L.off_slot);
-    s.split_units = reinterpret_cast<int4*>(ws + L.off_split);
-    s.n_split = reinterpret_cast<int32_t*>(ws) + 2;
-    s.split_grid = may_split ? grid_sm : 0;
-    s.n_units = reinterpret_cast<int32_t*>(ws);
-    s.lens_ok = reinterpret_cast<int32_t*>(ws) + 1;
-    s.err = d->err;
-    cudaError_t e = rr::launch_sched(s, stream);
-    if (e != cudaSuccess) return cuda_fail(e, "schedule kernel launch");
-    if (T == 0) return RR_OK;
-
-    rr::AttnArgs a;
-    memset(&a, 0, sizeof a);
-    if ((rc = encode_3d(&a.tm_q, q, (uint64_t)D, (uint64_t)Hq, (uint64_t)T, (uint64_t)D * 2, (uint64_t)Hq * D * 2, 64,
-                        (uint32_t)G, (uint32_t)tq)))
-        return rc;
-    const uint64_t rows = (uint64_t)dims->num_pages * (uint64_t)ps;
-    if ((rc = encode_2d(&a.tm_k, k_pool, (uint64_t)Hkv * D, rows, (uint64_t)Hkv * D * 2, 64, (uint32_t)ps))) return rc;
-    if ((rc = encode_2d(&a.tm_v, v_pool, (uint64_t)Hkv * D, rows, (uint64_t)Hkv * D * 2, 64, (uint32_t)ps))) return rc;
-    a.page_table = page_table;
-    a.prefix = prefix_lens;
-    a.suffix = suffix_lens;
-    a.cu = s.cu;
-    a.units = s.units;
-    a.n_units = s.n_units;
-    a.item_slot = s.item_slot;
-    a.part_o = reinterpret_cast<float*>(ws + L.off_o);
-    a.part_ml = reinterpret_cast<float2*>(ws + L.off_ml);
-    a.err = d->err;
-    a.out = out;
-    a.num_pages = dims->num_pages;
-    a.Hq = Hq;
-    a.G = G;
-    a.ps = ps;
-    a.max_pages = dims->max_pages;
-    a.tq = tq;
-    a.oob_row = (int32_t)rows;
-    const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)D);
-    a.scale_log2 = scale * 1.4426950408889634f;
-    const int64_t grid = std::min<int64_t>((int64_t)d->sm_count, max_items);
-    e = rr::launch_extend_attention(a, D, (int)std::max<int64_t>(grid, 1), stream);
-    if (e != cudaSuccess) return cuda_fail(e, "extend attention kernel launch");
-    if (may_split) {
-        rr::CombineArgs c;
-        c.split_units = s.split_units;
-        c.n_split = s.n_split;
-        c.part_o = a.part_o;
-        c.part_ml = a.part_ml;
-        c.suffix = suffix_lens;
-        c.cu = s.cu;
-        c.out = out;
-        c.Hq = Hq;
-        c.G = G;
-        c.D = D;
-        c.tq = tq;
-        e = rr::launch_combine(c, (int)max_split, stream);
-        if (e != cudaSuccess) return cuda_fail(e, "split-K combine kernel launch");
-    }
-    return RR_OK;
+int rr_decode_attention(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
+                        const int32_t* kv_lens, void* out, const rr_dims* dims, float softmax_scale,
+                        cudaStream_t stream) {
+    return attention_impl(q, k_pool, v_pool, page_table, nullptr, nullptr, kv_lens, out, dims, softmax_scale, stream,
+                          true);
 }
 
 int rr_validate_page_table(const int32_t* page_table, const int32_t* prefix_lens, const int32_t* suffix_lens,

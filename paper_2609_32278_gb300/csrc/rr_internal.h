@@ -93,5 +93,10 @@ cudaError_t launch_kv_append(const AppendArgs& a, int sm_count, cudaStream_t st)
 // Returns cudaErrorInvalidValue for an unsupported head dim.
 cudaError_t launch_extend_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st);
 size_t extend_attention_smem_bytes(int head_dim);
+// Decode: the same arguments (tm_q boxes one token of G heads); units from the schedule run on
+// prefix = kv_lens - 1 and suffix = 1, which launch_decode_lens writes.
+cudaError_t launch_decode_lens(const int32_t* kv_lens, int32_t* prefix, int32_t* suffix, int32_t B, int32_t* err,
+                               cudaStream_t st);
+cudaError_t launch_decode_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st);
 
 }  // namespace rr

@@ -143,6 +143,7 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
             atomicCAS(a.err, 0, RR_ERR_LENS);
             *a.lens_ok = 0;
             *a.n_units = 0;
+            if (a.n_split) *a.n_split = 0;  // the combine must not replay a previous call's split list
         }
         return;  // uniform: every thread sees the same `ok`
     }

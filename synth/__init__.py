@@ -281,6 +281,22 @@ def config(name: str, seed: int = 0, free_hbm_bytes: Optional[int] = None) -> Wo
 
 CONFIGS = ("c1_tiny", "c2_llama3_8b", "c3_lru", "c3_rr", "c4_coding", "c5_shared")
 
+# Decode batches: the agents of an extend workload one step later -- each agent's history after its
+# extend (P + S cached tokens) plus one new token (suffix 1), same heads, same shared prefix.
+DECODE_CONFIGS = ("c2_decode", "c4_decode", "c5_decode")
+_DECODE_BASE = {"c2_decode": "c2_llama3_8b", "c4_decode": "c4_coding", "c5_decode": "c5_shared"}
+
+
+def decode_config(name: str, seed: int = 0, free_hbm_bytes: Optional[int] = None) -> Workload:
+    """c2_decode: 32 agents, 32/8 heads, d128, keys = c2's P + S + 1 (~9k-35k)
+    c4_decode: 16 agents, 64/8 heads, d128, keys = c4's P + S + 1 (~130k-265k), pool as c4_coding
+    c5_decode: 128 agents, 32/8 heads, d128, keys = c5's P + S + 1, the 4096-token prefix shared by all"""
+    base = config(_DECODE_BASE[name], seed, free_hbm_bytes)
+    P = np.asarray(base.prefix_lens, dtype=np.int64) + np.asarray(base.suffix_lens, dtype=np.int64)
+    num_pages = base.num_pages if name == "c4_decode" else None
+    return custom(name, base.B, base.Hq, base.Hkv, base.D, P, np.ones(base.B, dtype=np.int64), ps=base.ps,
+                  shared_len=base.shared_len, num_pages=num_pages, seed=seed)
+
 
 # --------------------------------------------------------------------------- CPU tensors
 
