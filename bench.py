@@ -328,6 +328,85 @@ def decode_leg(args, rr, synth, dev, st, peaks, rank):
     return res
 
 
+# Replay leg: the policy's effect on per-request extend cost (Sec. 4's P99 metrics), with the attention
+# time of each request taken from a cost model fitted to this GPU's measured extend kernel.
+REPLAY_MODELS = {  # attention geometry of the two served models of Sec. 4
+    "conversational": {"model": "Qwen3-Coder-30B-A3B attention (32 q / 4 kv heads, d128)", "Hq": 32, "Hkv": 4},
+    "coding": {"model": "Qwen3-8B attention (32 q / 8 kv heads, d128)", "Hq": 32, "Hkv": 8},
+}
+# kind, agents, admitted concurrency, capacity as a fraction of the admitted agents' summed final contexts:
+# points inside the regime of Eq. 1 on these traces (active demand fits, live idle demand does not) --
+# at 0.6 and above nothing is evicted from live agents, far below it every policy thrashes
+REPLAY_SETTINGS = [
+    ("conversational", 222, 40, 0.4), ("conversational", 222, 80, 0.4), ("conversational", 222, 80, 0.6),
+    ("coding", 64, 16, 0.4), ("coding", 64, 16, 0.5), ("coding", 64, 32, 0.4),
+]
+REPLAY_POLICIES = [  # label, policy, completion signals
+    ("lru", "lru", False), ("lru+cs", "lru", True), ("rr-evict+cs", "rr", True), ("rr-tiered", "tiered", False),
+]
+
+
+def measure_extend_grid(rr, synth, dev, st, Hq, Hkv, D=128, reps=5):
+    """Median CUDA-event time of one agent's append + extend attention for a grid of (P, S)."""
+    import torch
+    out = []
+    for P in (0, 2048, 8192, 32768, 131072):
+        for S in (64, 256, 1024, 4096, 16384, 65536, 131072):
+            if P + S > 262144:
+                continue
+            wl = synth.custom(f"grid_{P}_{S}", 1, Hq, Hkv, D, [P], [S], seed=11)
+            g = synth.gpu_tensors(wl, dev)
+            args = (g["q"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"], g["suffix_lens"])
+            o = torch.empty_like(g["q"])
+            for _ in range(2):
+                rr.kv_append(g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                             g["suffix_lens"])
+                rr.extend_attention(*args, out=o)
+            ts = []
+            for _ in range(reps):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(st)
+                rr.kv_append(g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                             g["suffix_lens"])
+                rr.extend_attention(*args, out=o)
+                e1.record(st)
+                e1.synchronize()
+                ts.append(e0.elapsed_time(e1) * 1e-3)
+            if rr.device_error():
+                raise RuntimeError("device error in the replay cost grid")
+            out.append((P, S, statistics.median(ts)))
+            del g, o
+    torch.cuda.empty_cache()
+    return out
+
+
+def replay_leg(rr, synth, dev, st):
+    from paper_2609_32278_gb300 import policy as pol
+    res = {"note": ("synthetic agent traces (policy.synthetic_traces) replayed under each policy; attention "
+                    "time per request = c0 + c1 S + c2 F(P, S) + c3 (P + S) fitted to this GPU's measured "
+                    "single-agent append + extend time (one layer)"), "models": {}, "runs": []}
+    costs = {}
+    for kind, m in REPLAY_MODELS.items():
+        grid = measure_extend_grid(rr, synth, dev, st, m["Hq"], m["Hkv"])
+        cost, coef, rel = pol.fit_extend_cost(grid, m["Hq"], 128)
+        costs[kind] = cost
+        res["models"][kind] = {"model": m["model"], "coef_s_call_token_flop_key": coef,
+                               "fit_max_rel_err": rel, "grid_points": len(grid),
+                               "grid": [(P, S, round(t * 1e3, 4)) for P, S, t in grid]}
+    for kind, n, conc, frac in REPLAY_SETTINGS:
+        traces = pol.synthetic_traces(n, kind, seed=0)
+        finals = sorted(sum(t.new_tokens) + sum(t.output_tokens) for t in traces)
+        cap = int(frac * sum(finals[-conc:]))
+        run = {"workload": kind, "agents": n, "concurrency": conc, "capacity_tokens": cap,
+               "capacity_note": f"{frac} x the summed final contexts of the {conc} largest agents", "policies": {}}
+        for label, policy, cs in REPLAY_POLICIES:
+            reqs = pol.replay(traces, cap, policy, shared_prompt=2048, chunk=1024, completion_signals=cs,
+                              concurrency=conc)
+            run["policies"][label] = pol.summarize(reqs, costs[kind])
+        res["runs"].append(run)
+    return res
+
+
 def run_ours(args, world, rank, local):
     import torch
     import synth
@@ -434,6 +513,11 @@ def run_ours(args, world, rank, local):
     per_agent = None
     if args.per_agent:
         per_agent = per_agent_latency(rr, wl, g, dev, st)
+    replay = None
+    if args.replay and rank == 0:
+        g.clear()
+        torch.cuda.empty_cache()
+        replay = replay_leg(rr, synth, dev, st)
     decode = None
     if not args.no_decode:
         g.clear()
@@ -475,6 +559,8 @@ def run_ours(args, world, rank, local):
         line["per_agent_extend"] = per_agent
     if decode is not None:
         line["decode"] = decode
+    if replay is not None:
+        line["replay"] = replay
     if rank == 0 and not args.no_cpu_baseline:
         f, t, rows, threads = cpu_oracle_sample(wl, args.baseline_flops, seed=7)
         line["cpu_baseline"] = {"value": f / t / 1e12, "unit": "TFLOP/s", "cores": threads, "kind": "oracle",
@@ -501,6 +587,8 @@ def main():
     ap.add_argument("--decode-config", default="c2_decode", help="decode batch of the decode leg")
     ap.add_argument("--no-decode", action="store_true", help="skip the decode-attention leg")
     ap.add_argument("--decode-agents", type=int, default=0, help="only the first N agents of the decode batch")
+    ap.add_argument("--replay", action="store_true",
+                    help="also replay synthetic agent traces under each eviction policy (modelled attention TTFT)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -358,23 +358,32 @@ class Request:
 
 def replay(traces: List[AgentTrace], capacity: int, policy: str, shared_prompt: int = 0, chunk: int = 1024,
            page_size: int = 16, completion_signals: bool = True, tier_width: float = 1.0,
-           service_time_per_token: float = 1e-4) -> List[Request]:
+           service_time_per_token: float = 1e-4, concurrency: Optional[int] = None) -> List[Request]:
     """Replay agent traces against one prefix cache under `policy`; returns every request.
 
     Each turn: prefix match (refreshing recency), eviction of what the uncached
     part needs, insertion of prompt + output, an active period proportional to
     the uncached tokens, then the recorded idle gap.  A finished agent's unshared
     cache is released at once if `completion_signals`.
+
+    `concurrency` caps the admitted agents (Sec. 4's replay: the agent slots are
+    filled first, then a new agent is admitted only when a resident one exits;
+    an admitted agent stays admitted while idle between turns).  None admits
+    every trace at its start time.
     """
     cache = RadixCache(capacity, page_size)
     if shared_prompt:
         cache.add_shared_prefix(shared_prompt)
     events = []
     hist = {}
+    waiting = deque()
     for a, tr in enumerate(traces):
         cache.add_agent(a)
         hist[a] = shared_prompt
-        heapq.heappush(events, (tr.start, 0, a, 0))      # (time, kind 0=arrive 1=finish, agent, turn)
+        if concurrency is None or a < concurrency:
+            heapq.heappush(events, (tr.start, 0, a, 0))      # (time, kind 0=arrive 1=finish, agent, turn)
+        else:
+            waiting.append(a)
     out: List[Request] = []
     while events:
         now, kind, a, k = heapq.heappop(events)
@@ -383,8 +392,11 @@ def replay(traces: List[AgentTrace], capacity: int, policy: str, shared_prompt: 
             cache.set_active(a, False)
             if k + 1 < len(tr.new_tokens):
                 heapq.heappush(events, (now + tr.gaps[k], 0, a, k + 1))
-            elif completion_signals:
-                cache.complete(a)
+            else:
+                if completion_signals:
+                    cache.complete(a)
+                if waiting:  # the slot passes to the next agent in line
+                    heapq.heappush(events, (now, 0, waiting.popleft(), 0))
             continue
         prompt = hist[a] + tr.new_tokens[k]
         cached = cache.match(a, now)
@@ -401,6 +413,87 @@ def replay(traces: List[AgentTrace], capacity: int, policy: str, shared_prompt: 
         busy = service_time_per_token * (prompt - cached + tr.output_tokens[k])
         heapq.heappush(events, (now + busy, 1, a, k))
     return out
+
+
+# --------------------------------------------------------------------------- synthetic agent traces
+
+def synthetic_traces(n_agents: int, kind: str = "conversational", seed: int = 0) -> List[AgentTrace]:
+    """Seeded agent traces shaped like the paper's two workloads (Sec. 4), which are not available here.
+
+    conversational -- customer-service agents (the tau^2-bench banking shape): 8-30 turns; a first
+      user message of 300-1500 tokens, then per turn 100-1500 appended tokens (tool results or the
+      user's reply); 30-400 output tokens; after a tool call a short gap (0.5-4 s), after a reply
+      to the user a long pause (10-90 s) -- one turn in three waits for the user.
+    coding -- software-engineering agents (the SWE-bench shape): 15-60 turns; a first message of
+      1000-4000 tokens (issue + repository summary), then 300-6000 appended tokens per turn (file
+      views, test logs); 50-800 output tokens; gaps of 1-20 s (tool and test execution).
+    Agents start over the first 30 s.  Token counts are uniform on the ranges, gaps uniform on
+    theirs; every number comes from one seeded generator, none from any dataset.
+    """
+    import random
+    rnd = random.Random((seed * 1000003) ^ (0x5EED if kind == "coding" else 0xC0DE))
+    out = []
+    for _ in range(n_agents):
+        if kind == "conversational":
+            turns = rnd.randint(8, 30)
+            new = [rnd.randint(300, 1500)] + [rnd.randint(100, 1500) for _ in range(turns - 1)]
+            outs = [rnd.randint(30, 400) for _ in range(turns)]
+            gaps = [rnd.uniform(10.0, 90.0) if rnd.random() < 1 / 3 else rnd.uniform(0.5, 4.0) for _ in range(turns)]
+        elif kind == "coding":
+            turns = rnd.randint(15, 60)
+            new = [rnd.randint(1000, 4000)] + [rnd.randint(300, 6000) for _ in range(turns - 1)]
+            outs = [rnd.randint(50, 800) for _ in range(turns)]
+            gaps = [rnd.uniform(1.0, 20.0) for _ in range(turns)]
+        else:
+            raise ValueError(kind)
+        out.append(AgentTrace(new_tokens=new, output_tokens=outs, gaps=gaps, start=rnd.uniform(0.0, 30.0)))
+    return out
+
+
+def percentile(values, p: float) -> float:
+    """Nearest-rank percentile (p in [0, 100]) of a non-empty sequence."""
+    v = sorted(values)
+    k = max(0, min(len(v) - 1, int(-(-p * len(v) // 100)) - 1))
+    return float(v[k])
+
+
+def summarize(requests: List[Request], cost=None) -> Dict[str, float]:
+    """Sec. 4's per-request metrics: uncached prompt tokens (P50, P99, mean, max) and, given
+    cost(P, S) -> seconds, the modelled attention time of each request's extend (P50, P99, mean, max)."""
+    unc = [r.uncached for r in requests]
+    res = {"requests": len(requests), "uncached_p50": percentile(unc, 50), "uncached_p99": percentile(unc, 99),
+           "uncached_mean": sum(unc) / len(unc), "uncached_max": float(max(unc))}
+    if cost is not None:
+        t = [cost(r.cached, r.uncached) for r in requests]
+        res.update({"ttft_attn_p50_ms": 1e3 * percentile(t, 50), "ttft_attn_p99_ms": 1e3 * percentile(t, 99),
+                    "ttft_attn_mean_ms": 1e3 * sum(t) / len(t), "ttft_attn_max_ms": 1e3 * max(t)})
+    return res
+
+
+def fit_extend_cost(samples, Hq: int, D: int):
+    """Least-squares fit of t(P, S) = c0 + c1 S + c2 F(P, S) + c3 (P + S) to measured (P, S, seconds) samples,
+    weighted by 1/t (relative error).  F = 4 D Hq (S P + S (S + 1) / 2) is the extend attention's flops
+    (the tensor-bound part); P + S, the keys read, carries what flops miss when a short suffix over a long
+    prefix leaves few work units in flight.  Coefficients are clipped at zero.  Returns (cost function,
+    (c0, c1, c2, c3), max relative error over the samples)."""
+    import numpy as np
+
+    def feats(P, S):
+        return [1.0, float(S), 4.0 * D * Hq * (S * P + S * (S + 1) / 2.0), float(P + S)]
+
+    A = np.asarray([feats(P, S) for P, S, _ in samples])
+    y = np.asarray([t for _, _, t in samples])
+    w = 1.0 / y
+    coef, *_ = np.linalg.lstsq(A * w[:, None], y * w, rcond=None)
+    coef = np.maximum(coef, 0.0)
+
+    def cost(P, S):
+        if S <= 0:
+            return 0.0
+        return float(np.dot(coef, feats(P, S)))
+
+    rel = float(np.max(np.abs(A @ coef - y) / y))
+    return cost, tuple(float(c) for c in coef), rel
 
 
 def batch_lengths(requests: List[Request], batch: int, start: int = 0):

@@ -175,3 +175,81 @@ def test_replay_rr_cuts_the_uncached_tail():
         assert all(r.cached <= r.prompt_len for r in reqs)
     assert res["rr"][0] < res["lru"][0]      # P99 uncached tokens (Sec. 4 metric)
     assert res["rr"][2] < res["lru"][2]
+
+
+# ----------------------------------------------------------------------------- replay with admission, metrics
+
+def test_synthetic_traces_are_seeded_and_in_range():
+    a = pol.synthetic_traces(30, "conversational", seed=3)
+    b = pol.synthetic_traces(30, "conversational", seed=3)
+    c = pol.synthetic_traces(30, "conversational", seed=4)
+    assert [t.new_tokens for t in a] == [t.new_tokens for t in b]
+    assert [t.new_tokens for t in a] != [t.new_tokens for t in c]
+    for t in a:
+        assert 8 <= len(t.new_tokens) <= 30 and len(t.output_tokens) == len(t.gaps) == len(t.new_tokens)
+        assert 300 <= t.new_tokens[0] <= 1500 and all(100 <= x <= 1500 for x in t.new_tokens[1:])
+        assert all(0.5 <= g <= 90.0 for g in t.gaps)
+    for t in pol.synthetic_traces(10, "coding", seed=0):
+        assert 15 <= len(t.new_tokens) <= 60 and all(300 <= x <= 6000 for x in t.new_tokens[1:])
+    with pytest.raises(ValueError):
+        pol.synthetic_traces(1, "chat")
+
+
+def test_replay_never_admits_more_than_the_concurrency():
+    traces = pol.synthetic_traces(40, "coding", seed=1)
+    conc = 7
+    reqs = pol.replay(traces, 10 ** 9, "lru", concurrency=conc)
+    first, last = {}, {}
+    for r in reqs:
+        first.setdefault(r.agent, r.time)
+        last[r.agent] = r.time
+    assert len(first) == 40                            # every agent is eventually admitted
+    for r in reqs:
+        live = sum(1 for a in first if first[a] <= r.time <= last[a])
+        assert live <= conc
+    # with unbounded capacity every turn after the first reuses the whole previous context
+    by_agent = {}
+    for r in reqs:
+        by_agent.setdefault(r.agent, []).append(r)
+    for a, rs in by_agent.items():
+        for k in range(1, len(rs)):
+            assert rs[k].cached == rs[k - 1].prompt_len + traces[a].output_tokens[k - 1]
+
+
+def test_percentile_is_nearest_rank():
+    v = list(range(1, 101))
+    assert pol.percentile(v, 99) == 99 and pol.percentile(v, 50) == 50 and pol.percentile(v, 100) == 100
+    assert pol.percentile([5], 99) == 5 and pol.percentile([3, 1, 2], 0) == 1
+
+
+def test_fit_extend_cost_recovers_a_known_model():
+    c0, c1, c2, c3 = 2e-5, 3e-9, 1.0 / 1.3e15, 4e-9
+    model = lambda P, S: c0 + c1 * S + c2 * 4.0 * 128 * 32 * (S * P + S * (S + 1) / 2.0) + c3 * (P + S)
+    samples = [(P, S, model(P, S)) for P in (0, 1000, 8000, 64000) for S in (64, 512, 4096, 32000)]
+    cost, coef, rel = pol.fit_extend_cost(samples, 32, 128)
+    assert rel < 1e-6
+    assert coef[0] == pytest.approx(c0, rel=1e-4) and coef[2] == pytest.approx(c2, rel=1e-6)
+    assert coef[3] == pytest.approx(c3, rel=1e-4)
+    assert cost(1000, 512) == pytest.approx(model(1000, 512))
+    assert cost(500, 0) == 0.0
+
+
+def test_summarize_reports_the_sec4_metrics():
+    reqs = [pol.Request(0, k, float(k), 100 + k, 100 - k) for k in range(50)]
+    s = pol.summarize(reqs, cost=lambda P, S: 1e-3 * S)
+    assert s["requests"] == 50 and s["uncached_max"] == 2 * 49
+    assert s["uncached_p99"] == pol.percentile([2 * k for k in range(50)], 99)
+    assert s["ttft_attn_max_ms"] == pytest.approx(98.0)
+
+
+def test_rr_cuts_the_tail_on_the_synthetic_conversational_replay():
+    """Sec. 4's comparison on the seeded conversational traces, at a capacity inside Eq. 1's regime."""
+    traces = pol.synthetic_traces(222, "conversational", seed=0)
+    finals = sorted(sum(t.new_tokens) + sum(t.output_tokens) for t in traces)
+    cap = int(0.4 * sum(finals[-40:]))
+    p99 = {}
+    for label, policy, cs in (("lru", "lru", False), ("lru+cs", "lru", True), ("rr", "rr", True)):
+        reqs = pol.replay(traces, cap, policy, shared_prompt=2048, chunk=1024, completion_signals=cs,
+                          concurrency=40)
+        p99[label] = pol.summarize(reqs)["uncached_p99"]
+    assert p99["rr"] < p99["lru+cs"] < p99["lru"]
