@@ -214,8 +214,11 @@ int attention_impl(const void* q, const void* k_pool, const void* v_pool, const 
     // least Hkv * T / unit_tokens units, so larger batches never split and need no partial buffers.
     const int grid_sm = d->sm_count;
     const bool may_split = (int64_t)Hkv * (T / unit_tokens) < 2ll * grid_sm;
+    // Decode is bound by HBM and an item costs little beyond its bytes, so its splits aim at 6 waves
+    // (a short last wave); extend splits aim at 2 (fewer partial rows to write and merge).
+    const int split_waves = decode ? 6 : 2;
     const int64_t max_split = may_split ? 2ll * grid_sm : 0;
-    const int64_t slots = may_split ? 4ll * grid_sm : 0;
+    const int64_t slots = may_split ? (int64_t)(split_waves + 2) * grid_sm : 0;
     const int64_t max_items = std::max<int64_t>(max_units, slots);
     const Layout L = layout_for(B, max_items, max_split, slots, D, decode);
     if ((rc = ensure_ws(*d, L.total))) return rc;
@@ -248,6 +251,7 @@ int attention_impl(const void* q, const void* k_pool, const void* v_pool, const 
     s.split_units = reinterpret_cast<int4*>(ws + L.off_split);
     s.n_split = reinterpret_cast<int32_t*>(ws) + 2;
     s.split_grid = may_split ? grid_sm : 0;
+    s.split_waves = split_waves;
     s.n_units = reinterpret_cast<int32_t*>(ws);
     s.lens_ok = reinterpret_cast<int32_t*>(ws) + 1;
     s.err = d->err;

@@ -33,6 +33,7 @@ struct SchedArgs {
     int4* split_units;     // [units] split units for the combine: (agent, kv head | nsplit << 16, unit, first slot)
     int32_t* n_split;      // number of split units
     int32_t split_grid;    // persistent grid size; 0 disables splitting
+    int32_t split_waves;   // a split aims at this many waves of items (2 if 0); slots needed: (waves + 2) x grid
     int32_t* n_units;      // number of items
     int32_t* lens_ok;
     int32_t* err;

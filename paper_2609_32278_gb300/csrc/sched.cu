@@ -163,10 +163,11 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     const long long tot_cost = block_sum(my_cost, s_ws);
 
     // Split the KV range of every unit when the batch has fewer than two waves of units: a unit of
-    // `cost` KV tiles becomes ceil(cost / target) items (at most 64), target = total / (2 waves), at
-    // least 8 tiles.  Then items <= total/target + units <= 4 waves, which bounds the partial buffers.
+    // `cost` KV tiles becomes ceil(cost / target) items (at most 64), target = total / (W waves), at
+    // least 8 tiles.  Then items <= total/target + units <= (W + 2) waves, which bounds the partial buffers.
+    const long long W = a.split_waves > 0 ? a.split_waves : 2;
     const bool split = a.split_grid > 0 && tot_u < 2ll * a.split_grid && tot_u <= 1024 && tot_u > 0;
-    const long long target = split ? max(8ll, (tot_cost + 2ll * a.split_grid - 1) / (2ll * a.split_grid)) : 0;
+    const long long target = split ? max(8ll, (tot_cost + W * a.split_grid - 1) / (W * a.split_grid)) : 0;
     int my_b = 0, my_g = 0, my_u = 0, my_ns = 1;
     long long my_unit_cost = 0;
     if (split && tid < tot_u) {  // one unit per thread
