@@ -474,6 +474,27 @@ def run_ours(args, world, rank, local):
     value = world * F / (ms_step * 1e-3) / 1e12
     tok_s = world * wl.T / (ms_step * 1e-3)
 
+    # ---- the same step as one launch (rr_extend_step: append fused into the attention kernel)
+    fused = None
+    if not args.no_fused:
+        fev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+        for _ in range(args.warmup):
+            rr.extend_step(g["q"], g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"],
+                           g["prefix_lens"], g["suffix_lens"], out=g["out"])
+        torch.cuda.synchronize(dev)
+        for e0, e1 in fev:
+            e0.record(st)
+            rr.extend_step(g["q"], g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"],
+                           g["prefix_lens"], g["suffix_lens"], out=g["out"])
+            e1.record(st)
+        torch.cuda.synchronize(dev)
+        if rr.device_error():
+            raise RuntimeError("device error in the fused-step region")
+        f_ms = max_over_ranks(statistics.mean(e0.elapsed_time(e1) for e0, e1 in fev), world, dev)
+        fused = {"ms_per_step": f_ms, "value": world * F / (f_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
+                 "uncached_suffix_tokens_per_s": world * wl.T / (f_ms * 1e-3),
+                 "vs_two_calls": ms_step / f_ms}
+
     e2e = None
     if not args.no_e2e:
         # ---- end to end through the public API: every step copies its inputs from pinned host memory to
@@ -585,6 +606,8 @@ def run_ours(args, world, rank, local):
     }
     if per_agent is not None:
         line["per_agent_extend"] = per_agent
+    if fused is not None:
+        line["fused_step"] = fused
     if decode is not None:
         line["decode"] = decode
     if replay is not None:
@@ -614,6 +637,7 @@ def main():
     ap.add_argument("--per-agent", action="store_true", help="also time each agent's extend step alone")
     ap.add_argument("--decode-config", default="c2_decode", help="decode batch of the decode leg")
     ap.add_argument("--no-decode", action="store_true", help="skip the decode-attention leg")
+    ap.add_argument("--no-fused", action="store_true", help="skip the fused extend-step leg")
     ap.add_argument("--decode-agents", type=int, default=0, help="only the first N agents of the decode batch")
     ap.add_argument("--replay", action="store_true",
                     help="also replay synthetic agent traces under each eviction policy (modelled attention TTFT)")

@@ -112,6 +112,23 @@ int rr_extend_attention(const void* q, const void* k_pool, const void* v_pool, c
                         float softmax_scale, cudaStream_t stream);
 
 /*
+ * rr_extend_step -- the whole extend step of Sec. 2 in one attention launch:
+ * the same results as rr_kv_append followed by rr_extend_attention on the
+ * same stream (the pools receive the suffix K/V bit for bit, and `out` is
+ * bit-identical), without the separate pass over k_new / v_new.
+ *
+ * The attention kernel reads every suffix position's K/V straight from
+ * k_new / v_new [T][Hkv][D] (cached positions from the pool through
+ * page_table, as before), and each work unit also writes its own suffix rows
+ * into the pool slots page_table assigns to them, for later calls.  Arguments,
+ * layouts, preconditions and errors are those of the two calls it replaces;
+ * k_pool / v_pool are written, so they are non-const here.
+ */
+int rr_extend_step(const void* q, const void* k_new, const void* v_new, void* k_pool, void* v_pool,
+                   const int32_t* page_table, const int32_t* prefix_lens, const int32_t* suffix_lens, void* out,
+                   const rr_dims* dims, float softmax_scale, cudaStream_t stream);
+
+/*
  * rr_decode_attention -- decode attention over the same paged pool: the
  * extend attention above for a suffix of exactly one token per agent, the
  * step that follows an extend in an agent's turn (Sec. 2: an agent's request

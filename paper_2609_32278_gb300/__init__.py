@@ -35,7 +35,7 @@ RR_ERR_LENS = 6
 RR_ERR_OVERLAP = 7
 
 # Every symbol include/rr.h declares.
-EXPORTS = ("rr_kv_append", "rr_extend_attention", "rr_decode_attention", "rr_validate_page_table",
+EXPORTS = ("rr_kv_append", "rr_extend_attention", "rr_extend_step", "rr_decode_attention", "rr_validate_page_table",
            "rr_get_device_error", "rr_last_error", "rr_version", "rr_shutdown", "rr_extend_attention_noalloc")
 
 
@@ -73,6 +73,8 @@ def lib():
         L.rr_kv_append.argtypes = [vp, vp, vp, vp, vp, vp, vp, dp, vp]
         L.rr_extend_attention.restype = ctypes.c_int
         L.rr_extend_attention.argtypes = [vp, vp, vp, vp, vp, vp, vp, dp, ctypes.c_float, vp]
+        L.rr_extend_step.restype = ctypes.c_int
+        L.rr_extend_step.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, dp, ctypes.c_float, vp]
         L.rr_decode_attention.restype = ctypes.c_int
         L.rr_decode_attention.argtypes = [vp, vp, vp, vp, vp, vp, dp, ctypes.c_float, vp]
         L.rr_validate_page_table.restype = ctypes.c_int
@@ -169,6 +171,39 @@ def extend_attention(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, ou
     _check(lib().rr_extend_attention(q.data_ptr(), k_pool.data_ptr(), v_pool.data_ptr(), page_table.data_ptr(),
                                      prefix_lens.data_ptr(), suffix_lens.data_ptr(), out.data_ptr(),
                                      ctypes.byref(dims), float(softmax_scale), _stream_ptr(stream, q.device)))
+    return out
+
+
+def extend_step(q, k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens, out=None,
+                softmax_scale: float = 0.0, stream=None):
+    """kv_append + extend_attention in one attention launch (rr_extend_step): same pools, same output."""
+    import torch
+    _need(q, "q", torch.bfloat16, 3)
+    _need(k_new, "k_new", torch.bfloat16, 3)
+    _need(v_new, "v_new", torch.bfloat16, 3)
+    _need(k_pool, "k_pool", torch.bfloat16, 4)
+    _need(v_pool, "v_pool", torch.bfloat16, 4)
+    _need(page_table, "page_table", torch.int32, 2)
+    _need(prefix_lens, "prefix_lens", torch.int32, 1)
+    _need(suffix_lens, "suffix_lens", torch.int32, 1)
+    T, Hq, D = q.shape
+    num_pages, ps, Hkv, D2 = k_pool.shape
+    if v_pool.shape != k_pool.shape or D2 != D or k_new.shape != (T, Hkv, D) or v_new.shape != k_new.shape:
+        raise ValueError("q / k_new / v_new / pool shapes disagree")
+    B = prefix_lens.shape[0]
+    if suffix_lens.shape[0] != B or page_table.shape[0] != B:
+        raise ValueError("lens / page_table batch sizes disagree")
+    if out is None:
+        out = torch.empty_like(q)
+    else:
+        _need(out, "out", torch.bfloat16, 3)
+        if out.shape != q.shape:
+            raise ValueError("out must have q's shape")
+    dims = make_dims(B, Hq, Hkv, D, ps, page_table.shape[1], num_pages, T)
+    _check(lib().rr_extend_step(q.data_ptr(), k_new.data_ptr(), v_new.data_ptr(), k_pool.data_ptr(),
+                                v_pool.data_ptr(), page_table.data_ptr(), prefix_lens.data_ptr(),
+                                suffix_lens.data_ptr(), out.data_ptr(), ctypes.byref(dims), float(softmax_scale),
+                                _stream_ptr(stream, q.device)))
     return out
 
 

@@ -6,7 +6,8 @@
 //
 //   out[cu_b+i, h, :] = softmax_j( scale * q[cu_b+i, h, :] . K_j ) V_j,  j = 0 .. P_b + i
 //
-// Design (one persistent CTA per SM, 12 warps; warp 11 only lends its registers):
+// Design (one persistent CTA per SM, 12 warps; warp 11 only lends its registers, except in the
+// fused extend step, where it writes the suffix K/V into the pool):
 //   * work unit = (agent b, KV head g, kNQ = 2 consecutive Q tiles).  A Q tile
 //     packs 128/G suffix tokens x the G query heads that share KV head g into
 //     128 rows (GQA packing), so each K/V tile is loaded once for the whole
@@ -73,6 +74,7 @@ static_assert((2 * kRegsSoftmax + kRegsControl) * 32 <= 16384, "register split e
 constexpr int kWarpProducer = 8;
 constexpr int kWarpMMA = 9;
 constexpr int kWarpStage = 10;
+constexpr int kWarpAppend = 11;  // fused extend step: writes each unit's suffix K/V into the pool
 constexpr long long kWaitLimitCycles = 1ll << 33;  // ~4 s at 2 GHz
 
 template <int D, int NK, int NV>
@@ -90,7 +92,8 @@ struct Cfg {
     static constexpr int kKFull = 2, kKEmpty = 2 + NK, kVFull = 2 + 2 * NK, kVEmpty = 2 + 2 * NK + NV;
     static constexpr int kSFull = 2 + 2 * NK + 2 * NV, kPFull = kSFull + kNQ, kOFinal = kPFull + kNQ;
     static constexpr int kVTmp = kOFinal + kNQ, kDrain = kVTmp + 1, kDone = kDrain + 1;
-    static constexpr int kNumBars = kDone + 1;
+    static constexpr int kKTmp = kDone + 1;  // fused step: a K tile that needs fixing up before release
+    static constexpr int kNumBars = kKTmp + 1;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // u32 TMEM base, i32 abort flag
     static constexpr int kSmemBytes = kOffMisc + 16 + 1024;  // + slack to align the base to 1 KiB
     static_assert(kChunkBytes % 1024 == 0, "swizzle atoms must stay 1 KiB aligned");
@@ -167,7 +170,10 @@ __device__ __forceinline__ int unit_of(int wave, int cta, int grid) {
     return wave * grid + ((wave & 1) ? (grid - 1 - cta) : cta);
 }
 
-template <int D, int NK, int NV>
+// kFused: the one-launch extend step.  Suffix positions' K/V are read from k_new / v_new (the caller's
+// rows, not the pool), and warp 11 writes each work unit's own suffix rows into the pool, so no unit
+// waits for another CTA's pool writes; the attention result is bit-identical to append-then-attend.
+template <int D, int NK, int NV, bool kFused>
 __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_constant__ AttnArgs a) {
     using C = Cfg<D, NK, NV>;
     extern __shared__ uint8_t smem_raw[];
@@ -196,6 +202,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             ptx::mbar_init(bar(C::kOFinal + q), 1);
         }
         ptx::mbar_init(bar(C::kVTmp), 1);
+        ptx::mbar_init(bar(C::kKTmp), 1);
         ptx::mbar_init(bar(C::kDrain), 1);
         ptx::mbar_init(bar(C::kDone), 2 * kBM);  // every softmax thread, once, at its end
         *abort_flag = 0;
@@ -209,6 +216,10 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
         ptx::prefetch_tmap(&a.tm_q);
         ptx::prefetch_tmap(&a.tm_k);
         ptx::prefetch_tmap(&a.tm_v);
+        if constexpr (kFused) {
+            ptx::prefetch_tmap(&a.tm_knew);
+            ptx::prefetch_tmap(&a.tm_vnew);
+        }
     }
     ptx::tc_fence_before();
     __syncthreads();
@@ -224,9 +235,9 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
     if (warp == kWarpProducer) {
         // ------------------------------------------------------------ TMA producer
         const int ppt = kBN / a.ps;  // pages per KV tile (<= 16)
-        uint32_t kv_count = 0, unit_i = 0, vtmp_phase = 0;
+        uint32_t kv_count = 0, unit_i = 0, vtmp_phase = 0, ktmp_phase = 0;
         // copies in flight, for the abort drain: bit s of armed_* = stage s armed, bit s of par_* = its parity
-        int armed_q = -1, armed_vtmp = -1;
+        int armed_q = -1, armed_vtmp = -1, armed_ktmp = -1;
         uint32_t armed_k = 0, armed_v = 0, par_k = 0, par_v = 0;
         bool ok = true;
         for (int w = 0; ok; ++w) {
@@ -257,32 +268,48 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             for (int j = kb; j < ke; ++j, ++kv_count) {
                 const int sk = (int)(kv_count % NK), sv = (int)(kv_count % NV);
                 const uint32_t usek = kv_count / NK, usev = kv_count / NV;
-                int row = a.oob_row;  // page past the agent's keys: zero fill
+                // the page of this lane: from the pool, from k_new / v_new (a fused step's suffix
+                // positions), or past the agent's keys (a row past the pool: zero fill)
+                int row = a.oob_row;
+                bool from_new = false;
                 if (lane < ppt) {
                     const int lp = j * ppt + lane;
                     if (lp * a.ps < n_keys) {
-                        const int pid = a.page_table[(long long)b * a.max_pages + lp];
-                        if (pid >= 0 && (long long)pid < a.num_pages) row = pid * a.ps;
-                        else atomicCAS(a.err, 0, RR_ERR_OOB);
+                        if (kFused && lp * a.ps >= P) {
+                            from_new = true;
+                            row = cu_b + (lp * a.ps - P);
+                        } else {
+                            const int pid = a.page_table[(long long)b * a.max_pages + lp];
+                            if (pid >= 0 && (long long)pid < a.num_pages) row = pid * a.ps;
+                            else atomicCAS(a.err, 0, RR_ERR_OOB);
+                        }
                     }
                 }
+                // fused step, P in the middle of a page: that page comes from the pool and its slots
+                // from P on are rewritten from k_new / v_new in shared memory before the tiles are released
+                const bool straddle = kFused && (P % a.ps != 0) && (j == P / kBN);
                 // K tile
+                const uint32_t kbar = straddle ? bar(C::kKTmp) : bar(C::kKFull + sk);
                 if (lane == 0) {
                     if (usek > 0) ok = wait_bar(bar(C::kKEmpty + sk), (usek - 1) & 1, ctl);
-                    if (ok) ptx::mbar_arrive_expect_tx(bar(C::kKFull + sk), C::kKVTileBytes);
+                    if (ok) ptx::mbar_arrive_expect_tx(kbar, C::kKVTileBytes);
                 }
                 ok = __shfl_sync(0xffffffffu, ok, 0);
                 if (!ok) break;
-                armed_k |= 1u << sk;
-                par_k = (par_k & ~(1u << sk)) | ((usek & 1u) << sk);
+                if (!straddle) {
+                    armed_k |= 1u << sk;
+                    par_k = (par_k & ~(1u << sk)) | ((usek & 1u) << sk);
+                }
                 if (lane < ppt)
                     for (int c = 0; c < C::kChunks; ++c)
                         ptx::tma_load_2d(sb + C::kOffK + sk * C::kKVTileBytes + c * C::kChunkBytes + lane * a.ps * 128,
-                                         &a.tm_k, g * D + c * 64, row, bar(C::kKFull + sk));
-                // V tile; if the agent's last page is only partly its own, land it on the
-                // side barrier, clear the foreign slots, then release it to the MMA warp.
-                const bool clear_tail = (j == n_kv - 1) && (last_page_end > agent_len);
-                const uint32_t vbar = clear_tail ? bar(C::kVTmp) : bar(C::kVFull + sv);
+                                         from_new ? &a.tm_knew : &a.tm_k, g * D + c * 64, row, kbar);
+                // V tile; if the agent's last page is only partly its own (unfused), land it on the side
+                // barrier, clear the foreign slots, then release it to the MMA warp.  (A fused step reads
+                // a partial last page from v_new, whose rows past the agent are other agents' finite
+                // values or zero fill, unless it is the straddling page, which is rewritten anyway.)
+                const bool clear_tail = !kFused && (j == n_kv - 1) && (last_page_end > agent_len);
+                const uint32_t vbar = (clear_tail || straddle) ? bar(C::kVTmp) : bar(C::kVFull + sv);
                 if (lane == 0) {
                     if (usev > 0) ok = wait_bar(bar(C::kVEmpty + sv), (usev - 1) & 1, ctl);
                     if (ok) ptx::mbar_arrive_expect_tx(vbar, C::kKVTileBytes);
@@ -292,7 +319,47 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                 if (lane < ppt)
                     for (int c = 0; c < C::kChunks; ++c)
                         ptx::tma_load_2d(sb + C::kOffV + sv * C::kKVTileBytes + c * C::kChunkBytes + lane * a.ps * 128,
-                                         &a.tm_v, g * D + c * 64, row, vbar);
+                                         from_new ? &a.tm_vnew : &a.tm_v, g * D + c * 64, row, vbar);
+                if constexpr (kFused) {
+                    if (straddle) {
+                        // positions P .. end of P's page: rows r0 .. r1 of the tile, rewritten from the
+                        // agent's k_new / v_new rows (zeros past the agent's end), in the 128-byte swizzled
+                        // layout TMA wrote (16-byte unit u of row r sits at unit u ^ (r & 7))
+                        const int r0 = P - j * kBN, r1 = min(((P / a.ps) + 1) * a.ps - j * kBN, kBN);
+                        const int per_row = C::kChunks * 8;
+                        armed_ktmp = (int)ktmp_phase;
+                        armed_vtmp = (int)vtmp_phase;
+                        for (int kv = 0; kv < 2 && ok; ++kv) {
+                            const uint32_t tb = kv == 0 ? bar(C::kKTmp) : bar(C::kVTmp);
+                            if (lane == 0) ok = wait_bar(tb, kv == 0 ? ktmp_phase : vtmp_phase, ctl);
+                            ok = __shfl_sync(0xffffffffu, ok, 0);
+                            if (!ok) break;
+                            if (kv == 0) {
+                                armed_ktmp = -1;
+                                ktmp_phase ^= 1u;
+                            } else {
+                                armed_vtmp = -1;
+                                vtmp_phase ^= 1u;
+                            }
+                            uint8_t* tile = smem + (kv == 0 ? C::kOffK + sk * C::kKVTileBytes
+                                                            : C::kOffV + sv * C::kKVTileBytes);
+                            const uint4* src = kv == 0 ? a.knew : a.vnew;
+                            for (int e = lane; e < (r1 - r0) * per_row; e += 32) {
+                                const int r = r0 + e / per_row, c = (e / 8) % C::kChunks, v = e % 8;
+                                const int pos = j * kBN + r;
+                                uint4 val = make_uint4(0u, 0u, 0u, 0u);
+                                if (pos < agent_len)
+                                    val = src[(long long)(cu_b + pos - P) * a.row16 + (g * D + c * 64) / 8 + v];
+                                *reinterpret_cast<uint4*>(tile + c * C::kChunkBytes + r * 128 + ((v ^ (r & 7)) << 4)) = val;
+                            }
+                            ptx::fence_proxy_async_smem();
+                            __syncwarp();
+                            if (lane == 0) ptx::mbar_arrive(kv == 0 ? bar(C::kKFull + sk) : bar(C::kVFull + sv));
+                        }
+                        if (!ok) break;
+                        continue;
+                    }
+                }
                 if (clear_tail) {
                     armed_vtmp = (int)vtmp_phase;
                     if (lane == 0) ok = wait_bar(bar(C::kVTmp), vtmp_phase, ctl);
@@ -319,6 +386,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
         if (!ok && lane == 0) {  // abort: let every copy this warp started land before exit
             if (armed_q >= 0) drain_bar(bar(C::kQFull), (uint32_t)armed_q);
             if (armed_vtmp >= 0) drain_bar(bar(C::kVTmp), (uint32_t)armed_vtmp);
+            if (armed_ktmp >= 0) drain_bar(bar(C::kKTmp), (uint32_t)armed_ktmp);
             for (int s = 0; s < NK; ++s)
                 if (armed_k >> s & 1u) drain_bar(bar(C::kKFull + s), par_k >> s & 1u);
             for (int s = 0; s < NV; ++s)
@@ -467,6 +535,44 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
         __syncwarp();
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem, 512);
+    } else if (kFused && warp == kWarpAppend) {
+        // ------------------------------------------------------------ pool writer (fused step)
+        // Each work unit's own suffix rows of its KV head go to the agent's pool slots (every (token,
+        // KV head) belongs to exactly one unit; one piece of a split unit writes).  The kernel reads
+        // suffix K/V from k_new / v_new, so nothing waits for these writes: they are for later calls.
+        // Two tokens per pass (16 lanes each at D = 128, 8 at D = 64: one 16-byte vector of K and one
+        // of V per lane), page and slot by shifts (page sizes are powers of two): the loop stays
+        // light, since this warp shares its scheduler with two softmax warps.
+        constexpr int kPerTok = D / 8;      // 16-byte vectors of one head's row
+        constexpr int kTokPerPass = 32 / kPerTok;
+        const int ps_shift = __ffs(a.ps) - 1;
+        const int sub = lane / kPerTok, v = lane % kPerTok;
+        for (int w = 0;; ++w) {
+            const int ui = unit_of(w, cta, grid);
+            if (ui >= n_units) break;
+            const int4 U = a.units[ui];
+            if (((U.y >> 8) & 0xFF) != 0) continue;
+            const int b = U.x, g = U.y & 0xFF, u = U.z;
+            const int P = a.prefix[b], S = a.suffix[b], cu_b = a.cu[b];
+            const int t0 = u * unit_tokens, n = min(unit_tokens, S - t0);
+            const int32_t* pt = a.page_table + (long long)b * a.max_pages;
+            for (int tt = 0; tt < n; tt += kTokPerPass) {
+                const int t = tt + sub;
+                if (t >= n) continue;
+                const int pos = P + t0 + t;
+                const int pid = pt[pos >> ps_shift];
+                if (pid < 0 || (long long)pid >= a.num_pages) {
+                    atomicCAS(a.err, 0, RR_ERR_OOB);
+                    continue;
+                }
+                const long long src = (long long)(cu_b + t0 + t) * a.row16 + g * kPerTok + v;
+                const long long dst = (((long long)pid << ps_shift) + (pos & (a.ps - 1))) * a.row16 + g * kPerTok + v;
+                const uint4 kx = __ldcs(a.knew + src);
+                const uint4 vx = __ldcs(a.vnew + src);
+                a.kpool[dst] = kx;
+                a.vpool[dst] = vx;
+            }
+        }
     }
     return;
     }
@@ -638,7 +744,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
     ptx::mbar_arrive(bar(C::kDone));
 }
 
-template <int D, int NK, int NV>
+template <int D, int NK, int NV, bool kFused>
 cudaError_t launch_cfg(const AttnArgs& a, int grid, cudaStream_t st) {
     using C = Cfg<D, NK, NV>;
     static bool attr_done[64] = {};
@@ -647,12 +753,12 @@ cudaError_t launch_cfg(const AttnArgs& a, int grid, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     if (!attr_done[dev]) {
-        e = cudaFuncSetAttribute(extend_attn_kernel<D, NK, NV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(extend_attn_kernel<D, NK, NV, kFused>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  C::kSmemBytes);
         if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
-    extend_attn_kernel<D, NK, NV><<<grid, kThreads, C::kSmemBytes, st>>>(a);
+    extend_attn_kernel<D, NK, NV, kFused><<<grid, kThreads, C::kSmemBytes, st>>>(a);
     return cudaGetLastError();
 }
 
@@ -664,9 +770,9 @@ size_t extend_attention_smem_bytes(int head_dim) {
     return 0;
 }
 
-cudaError_t launch_extend_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st) {
-    if (head_dim == 128) return launch_cfg<128, 2, 3>(a, grid, st);
-    if (head_dim == 64) return launch_cfg<64, 4, 4>(a, grid, st);
+cudaError_t launch_extend_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st, bool fused) {
+    if (head_dim == 128) return fused ? launch_cfg<128, 2, 3, true>(a, grid, st) : launch_cfg<128, 2, 3, false>(a, grid, st);
+    if (head_dim == 64) return fused ? launch_cfg<64, 4, 4, true>(a, grid, st) : launch_cfg<64, 4, 4, false>(a, grid, st);
     return cudaErrorInvalidValue;
 }
 

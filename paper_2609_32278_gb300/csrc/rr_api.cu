@@ -174,15 +174,23 @@ int encode_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64
 
 namespace {
 
-// Extend attention, or decode attention (decode = true: kv_lens in place of the prefix / suffix lengths,
-// one query token per agent, the decode kernel in place of the extend kernel).
+// Extend attention; decode attention (decode = true: kv_lens in place of the prefix / suffix lengths,
+// one query token per agent, the decode kernel in place of the extend kernel); or the fused extend
+// step (k_new / v_new non-null: the extend kernel reads the suffix K/V from them and writes them into
+// the pools itself).
 int attention_impl(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
                    const int32_t* prefix_lens, const int32_t* suffix_lens, const int32_t* kv_lens, void* out,
-                   const rr_dims* dims, float softmax_scale, cudaStream_t stream, bool decode) {
+                   const rr_dims* dims, float softmax_scale, cudaStream_t stream, bool decode,
+                   const void* k_new = nullptr, const void* v_new = nullptr) {
     g_msg[0] = 0;
     int rc = check_dims(dims, true);
     if (rc) return rc;
     if (dims->total_tokens == 0 && dims->batch == 0) return RR_OK;
+    const bool fused = k_new != nullptr || v_new != nullptr;
+    if (fused) {
+        if (!k_new || !v_new) return fail(RR_ERR_INVALID_ARG, "the fused step needs both k_new and v_new");
+        if (!aligned16(k_new) || !aligned16(v_new)) return fail(RR_ERR_INVALID_ARG, "k_new / v_new must be 16-byte aligned");
+    }
     if (decode) {
         if (!page_table || !kv_lens) return fail(RR_ERR_INVALID_ARG, "null kv_lens or page table");
         if (dims->total_tokens != dims->batch)
@@ -289,8 +297,19 @@ int attention_impl(const void* q, const void* k_pool, const void* v_pool, const 
     const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)D);
     a.scale_log2 = scale * 1.4426950408889634f;
     const int64_t grid = std::min<int64_t>((int64_t)d->sm_count, max_items);
+    if (fused) {
+        // k_new / v_new [T][Hkv][D]: one row of Hkv * D per suffix token, the pool maps' box
+        const uint64_t row_elems = (uint64_t)Hkv * D;
+        if ((rc = encode_2d(&a.tm_knew, k_new, row_elems, (uint64_t)T, row_elems * 2, 64, (uint32_t)ps))) return rc;
+        if ((rc = encode_2d(&a.tm_vnew, v_new, row_elems, (uint64_t)T, row_elems * 2, 64, (uint32_t)ps))) return rc;
+        a.knew = static_cast<const uint4*>(k_new);
+        a.vnew = static_cast<const uint4*>(v_new);
+        a.kpool = static_cast<uint4*>(const_cast<void*>(k_pool));
+        a.vpool = static_cast<uint4*>(const_cast<void*>(v_pool));
+        a.row16 = (int32_t)(row_elems * 2 / 16);
+    }
     e = decode ? rr::launch_decode_attention(a, D, (int)std::max<int64_t>(grid, 1), stream)
-               : rr::launch_extend_attention(a, D, (int)std::max<int64_t>(grid, 1), stream);
+               : rr::launch_extend_attention(a, D, (int)std::max<int64_t>(grid, 1), stream, fused);
     if (e != cudaSuccess) return cuda_fail(e, decode ? "decode attention kernel launch" : "extend attention kernel launch");
     if (may_split) {
         rr::CombineArgs c;
@@ -396,6 +415,16 @@ int rr_decode_attention(const void* q, const void* k_pool, const void* v_pool, c
                         cudaStream_t stream) {
     return attention_impl(q, k_pool, v_pool, page_table, nullptr, nullptr, kv_lens, out, dims, softmax_scale, stream,
                           true);
+}
+
+int rr_extend_step(const void* q, const void* k_new, const void* v_new, void* k_pool, void* v_pool,
+                   const int32_t* page_table, const int32_t* prefix_lens, const int32_t* suffix_lens, void* out,
+                   const rr_dims* dims, float softmax_scale, cudaStream_t stream) {
+    if (dims && dims->total_tokens > 0 && (!k_new || !v_new))
+        return fail(RR_ERR_INVALID_ARG, "null k_new / v_new");
+    return attention_impl(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, nullptr, out, dims, softmax_scale,
+                          stream, false, dims && dims->total_tokens > 0 ? k_new : nullptr,
+                          dims && dims->total_tokens > 0 ? v_new : nullptr);
 }
 
 int rr_validate_page_table(const int32_t* page_table, const int32_t* prefix_lens, const int32_t* suffix_lens,

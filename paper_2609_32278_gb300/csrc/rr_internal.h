@@ -75,6 +75,14 @@ struct AttnArgs {
     int32_t tq;            // tokens per Q tile = 128 / G
     int32_t oob_row;       // first row past the pool (TMA fills it with zeros)
     float scale_log2;      // softmax scale * log2(e)
+    // fused extend step only (the suffix K/V is read from k_new / v_new and written to the pool here)
+    CUtensorMap tm_knew;   // k_new [T][Hkv*D], box {64, ps}, 128B swizzle
+    CUtensorMap tm_vnew;   // v_new, same
+    const uint4* knew;     // k_new / v_new rows and pool rows, 16-byte vectors
+    const uint4* vnew;
+    uint4* kpool;
+    uint4* vpool;
+    int32_t row16;         // 16-byte vectors per token row (Hkv * D * 2 / 16)
 };
 
 struct CombineArgs {
@@ -91,8 +99,9 @@ struct CombineArgs {
 cudaError_t launch_sched(const SchedArgs& a, cudaStream_t st);
 cudaError_t launch_combine(const CombineArgs& a, int grid, cudaStream_t st);
 cudaError_t launch_kv_append(const AppendArgs& a, int sm_count, cudaStream_t st);
-// Returns cudaErrorInvalidValue for an unsupported head dim.
-cudaError_t launch_extend_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st);
+// Returns cudaErrorInvalidValue for an unsupported head dim.  fused: the one-launch extend step (the
+// suffix K/V come from k_new / v_new, and the kernel also writes them into the pool).
+cudaError_t launch_extend_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st, bool fused = false);
 size_t extend_attention_smem_bytes(int head_dim);
 // Decode: the same arguments (tm_q boxes one token of G heads); units from the schedule run on
 // prefix = kv_lens - 1 and suffix = 1, which launch_decode_lens writes.
