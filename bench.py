@@ -630,7 +630,7 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--config", default="c2_llama3_8b")
     ap.add_argument("--ref-flops", type=float, default=1e10, help="oracle flops per reference-arm step")
-    ap.add_argument("--baseline-flops", type=float, default=6e10, help="oracle flops of the cpu_baseline sample")
+    ap.add_argument("--baseline-flops", type=float, default=3e11, help="oracle flops of the cpu_baseline sample (~10 s on 16 cores)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--agents", type=int, default=0, help="only the first N agents (small profiling case)")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
