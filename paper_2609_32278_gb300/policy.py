@@ -34,7 +34,7 @@ Policies
   describes but does not evaluate it.
 * ``complete``: a completion signal frees the agent's unshared cache at once.
 
-Readings where the paper is silent (listed again in the design doc):
+Readings where the paper is silent:
 * queue order at the start of a reclamation: least recently accessed first,
   ties by agent id;
 * SelectTailChunk frees min(chunk, leaf length, remaining demand rounded up to
