@@ -501,6 +501,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                         p_phase ^= 1u << q;
                         ptx::tc_fence_after();
                         issue_pv(q, sv, j > 0);
+                        if (q == kNQ - 1) ptx::mma_commit(bar(C::kVEmpty + sv));  // V(j) read by both PVs
                         if (!more) {
                             ptx::mma_commit(bar(C::kOFinal + q));
                             continue;
@@ -512,7 +513,6 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                         if (q == kNQ - 1) ptx::mma_commit(bar(C::kKEmpty + sk1));
                     }
                     if (!ok) break;
-                    ptx::mma_commit(bar(C::kVEmpty + sv));
                 }
                 if (!ok) break;
                 ptx::mma_commit(bar(C::kQEmpty));
