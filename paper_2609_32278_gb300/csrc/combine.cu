@@ -39,11 +39,15 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const CombineA
             const int tok = u * unit_tokens + q * a.tq + rr / a.G;
             if (tok >= S) continue;
             const int head = g * a.G + rr % a.G;
+            // Both passes are unrolled so the loads of several pieces are in flight together (the merge
+            // is a chain of dependent global loads otherwise: ~2 x nsplit memory latencies per row).
             float M = -INFINITY;
+#pragma unroll 8
             for (int s = 0; s < ns; ++s) M = fmaxf(M, a.part_ml[(long long)(base + s) * (kNQ * kBM) + row].x);
             float L = 0.f, acc[kPer];
 #pragma unroll
             for (int i = 0; i < kPer; ++i) acc[i] = 0.f;
+#pragma unroll 4
             for (int s = 0; s < ns; ++s) {
                 const long long prow = (long long)(base + s) * (kNQ * kBM) + row;
                 const float2 ml = a.part_ml[prow];

@@ -36,7 +36,8 @@
 //     the softmax works on tile t-1.
 //
 // The work items and their split-K pieces come from the same on-device
-// schedule as extend attention (one unit per agent and KV head), and a split
+// schedule as extend attention (one unit per agent and KV head; the schedule
+// also writes the lengths as prefix = L - 1, suffix = 1), and a split
 // item's partial uses the same layout (rows 0..G-1 of the unit), so the same
 // combine kernel merges them.
 //
@@ -200,6 +201,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + C::kOffMisc);
+    ptx::griddep_wait();  // the schedule kernel's output (launched as its dependent)
     const int n_units = *a.n_units;
     const int grid = gridDim.x, cta = blockIdx.x;
 
@@ -548,17 +550,6 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
     ptx::mbar_arrive(bar(C::kDone));
 }
 
-// prefix = L - 1 and suffix = 1 per agent: the decode batch in the lengths form the schedule reads
-__global__ void decode_lens_kernel(const int32_t* kv_lens, int32_t* prefix, int32_t* suffix, int32_t B,
-                                   int32_t* err) {
-    for (int b = blockIdx.x * blockDim.x + threadIdx.x; b < B; b += gridDim.x * blockDim.x) {
-        const int L = kv_lens[b];
-        if (L < 1) atomicCAS(err, 0, RR_ERR_LENS);
-        prefix[b] = L - 1;
-        suffix[b] = 1;
-    }
-}
-
 template <int D, int NS, int G>
 cudaError_t launch_dec(const AttnArgs& a, int grid, cudaStream_t st) {
     using C = DecCfg<D, NS>;
@@ -573,8 +564,7 @@ cudaError_t launch_dec(const AttnArgs& a, int grid, cudaStream_t st) {
         if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
-    decode_attn_kernel<D, NS, G><<<grid, kDecThreads, C::kSmemBytes, st>>>(a);
-    return cudaGetLastError();
+    return launch_after_sched(decode_attn_kernel<D, NS, G>, dim3(grid), dim3(kDecThreads), C::kSmemBytes, st, a);
 }
 
 template <int D, int NS>
@@ -590,13 +580,6 @@ cudaError_t launch_dec_g(const AttnArgs& a, int grid, cudaStream_t st) {
 }
 
 }  // namespace
-
-cudaError_t launch_decode_lens(const int32_t* kv_lens, int32_t* prefix, int32_t* suffix, int32_t B, int32_t* err,
-                               cudaStream_t st) {
-    if (B <= 0) return cudaSuccess;
-    decode_lens_kernel<<<(B + 255) / 256, 256, 0, st>>>(kv_lens, prefix, suffix, B, err);
-    return cudaGetLastError();
-}
 
 cudaError_t launch_decode_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st) {
     if (head_dim == 128) return launch_dec_g<128, 3>(a, grid, st);

@@ -225,6 +225,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + C::kOffMisc);
+    ptx::griddep_wait();  // the schedule kernel's output (launched as its dependent)
     const int n_units = *a.n_units;
     const int grid = gridDim.x, cta = blockIdx.x;
     const int unit_tokens = kNQ * a.tq;
@@ -758,8 +759,7 @@ cudaError_t launch_cfg(const AttnArgs& a, int grid, cudaStream_t st) {
         if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
-    extend_attn_kernel<D, NK, NV, kFused><<<grid, kThreads, C::kSmemBytes, st>>>(a);
-    return cudaGetLastError();
+    return launch_after_sched(extend_attn_kernel<D, NK, NV, kFused>, dim3(grid), dim3(kThreads), C::kSmemBytes, st, a);
 }
 
 }  // namespace

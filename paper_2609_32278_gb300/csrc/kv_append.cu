@@ -12,6 +12,7 @@
 // of traffic, bound by HBM bandwidth.  The suffix rows are read once
 // (streaming loads); the pool writes keep the default policy because the
 // attention kernel reads those pages right after.
+#include "ptx.cuh"
 #include "rr_internal.h"
 
 namespace rr {
@@ -30,6 +31,7 @@ __device__ __forceinline__ int last_le(const int32_t* off, int n, long long x) {
 constexpr int kAppendThreads = 256;
 
 __global__ void __launch_bounds__(kAppendThreads) kv_append_kernel(const AppendArgs a) {
+    ptx::griddep_wait();  // the schedule kernel's output (launched as its dependent)
     if (*a.lens_ok == 0) return;
     const int lane = threadIdx.x & 31;
     const long long warps = (long long)gridDim.x * (kAppendThreads / 32);
@@ -73,7 +75,8 @@ cudaError_t launch_kv_append(const AppendArgs& a, int sm_count, cudaStream_t st)
     const long long cap = (long long)sm_count * 8;  // 8 resident blocks of 256 threads per SM
     if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
-    kv_append_kernel<<<(unsigned)blocks, kAppendThreads, 0, st>>>(a);
+    cudaError_t e = launch_after_sched(kv_append_kernel, dim3((unsigned)blocks), dim3(kAppendThreads), 0, st, a);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 

@@ -232,18 +232,19 @@ int attention_impl(const void* q, const void* k_pool, const void* v_pool, const 
     if ((rc = ensure_ws(*d, L.total))) return rc;
     uint8_t* ws = static_cast<uint8_t*>(d->ws);
     cudaError_t e = cudaSuccess;
-    if (decode) {
-        int32_t* pre = reinterpret_cast<int32_t*>(ws + L.off_lens);
-        int32_t* suf = reinterpret_cast<int32_t*>(ws + L.off_lens + align256((size_t)B * 4));
-        e = rr::launch_decode_lens(kv_lens, pre, suf, (int32_t)B, d->err, stream);
-        if (e != cudaSuccess) return cuda_fail(e, "decode lengths kernel launch");
-        prefix_lens = pre;
-        suffix_lens = suf;
+    if (decode) {  // the schedule writes the lengths in prefix / suffix form itself
+        prefix_lens = reinterpret_cast<int32_t*>(ws + L.off_lens);
+        suffix_lens = reinterpret_cast<int32_t*>(ws + L.off_lens + align256((size_t)B * 4));
     }
 
     rr::SchedArgs s{};
     s.prefix = prefix_lens;
     s.suffix = suffix_lens;
+    if (decode) {
+        s.kv_lens = kv_lens;
+        s.prefix_out = const_cast<int32_t*>(prefix_lens);
+        s.suffix_out = const_cast<int32_t*>(suffix_lens);
+    }
     s.B = (int32_t)B;
     s.Hkv = Hkv;
     s.unit_tokens = unit_tokens;

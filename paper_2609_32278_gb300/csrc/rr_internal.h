@@ -19,6 +19,11 @@ constexpr int kCostBuckets = 4096;  // schedule: counting sort on the number of 
 struct SchedArgs {
     const int32_t* prefix;
     const int32_t* suffix;
+    // decode: when kv_lens is set, the schedule first writes prefix = kv_lens - 1 and suffix = 1 into
+    // the two arrays below (which prefix / suffix then point to) and flags kv_lens < 1
+    const int32_t* kv_lens;
+    int32_t* prefix_out;
+    int32_t* suffix_out;
     int32_t B, Hkv;
     int32_t unit_tokens;   // suffix tokens covered by one work unit (kNQ * kBM / G)
     int64_t T;
@@ -96,6 +101,25 @@ struct CombineArgs {
     int32_t Hq, G, D, tq;
 };
 
+// Launch `kernel` so that it may start while the schedule kernel before it on the stream finishes
+// (programmatic dependent launch); the kernel must call ptx::griddep_wait() before it reads anything
+// the schedule writes.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_after_sched(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                               Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
 cudaError_t launch_sched(const SchedArgs& a, cudaStream_t st);
 cudaError_t launch_combine(const CombineArgs& a, int grid, cudaStream_t st);
 cudaError_t launch_kv_append(const AppendArgs& a, int sm_count, cudaStream_t st);
@@ -104,9 +128,7 @@ cudaError_t launch_kv_append(const AppendArgs& a, int sm_count, cudaStream_t st)
 cudaError_t launch_extend_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st, bool fused = false);
 size_t extend_attention_smem_bytes(int head_dim);
 // Decode: the same arguments (tm_q boxes one token of G heads); units from the schedule run on
-// prefix = kv_lens - 1 and suffix = 1, which launch_decode_lens writes.
-cudaError_t launch_decode_lens(const int32_t* kv_lens, int32_t* prefix, int32_t* suffix, int32_t B, int32_t* err,
-                               cudaStream_t st);
+// prefix = kv_lens - 1 and suffix = 1, which the schedule writes (SchedArgs::kv_lens).
 cudaError_t launch_decode_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st);
 
 }  // namespace rr

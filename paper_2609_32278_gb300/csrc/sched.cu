@@ -17,6 +17,7 @@
 //      policy creates, Sec. 3.1-3.3).
 // Within a cost bucket the order is not fixed (atomics), which is harmless: a
 // unit's result does not depend on which CTA computes it or when.
+#include "ptx.cuh"
 #include "rr_internal.h"
 
 namespace rr {
@@ -31,6 +32,13 @@ __device__ __forceinline__ int last_le(const int32_t* off, int n, long long x) {
         if ((long long)off[mid] <= x) lo = mid; else hi = mid - 1;
     }
     return lo;
+}
+
+// KV tiles of piece sp of a unit of `cost` tiles split into ns pieces: floor((sp+1) cost / ns) -
+// floor(sp cost / ns), in 32-bit arithmetic (cost < 2^24, ns <= 64: the products stay below 2^31;
+// 64-bit division is a long software sequence, and this runs once per item in two passes).
+__device__ __forceinline__ int piece_tiles(int cost, int ns, int sp) {
+    return (sp + 1) * cost / ns - sp * cost / ns;
 }
 
 // Sum over the 1024 threads of the block (every thread gets the total).
@@ -81,11 +89,19 @@ __device__ void block_exclusive_scan2(long long x, long long y, long long& ex, l
     __syncthreads();
 }
 
+// Batches of at most this many agents keep their lengths and unit offsets in shared memory after the
+// first pass (every later pass, and the binary searches over the unit offsets, would otherwise be
+// chains of dependent global loads); larger batches read them from global memory.
+constexpr int kSchedSmemAgents = 2048;
+
 __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     __shared__ long long s_ws[32], s_wu[32];
     __shared__ int s_hist[kCostBuckets];
     __shared__ int s_bad;
+    extern __shared__ int32_t s_dyn[];  // [prefix: B][suffix: B][unit offsets: B + 1] when staged
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    // the consumer kernel may start its prologue now; it waits for this kernel before reading its output
+    ptx::griddep_launch_dependents();
     if (tid == 0) s_bad = 0;
     __syncthreads();
 
@@ -93,16 +109,34 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     const int B = a.B;
     const int chunk = (B + 1023) / 1024;
     const int b0 = min(B, tid * chunk), b1 = min(B, b0 + chunk);
+    if (a.kv_lens) {  // decode: the lengths in prefix / suffix form (read back below by the same threads,
+                      // and by every thread after the next barrier)
+        for (int b = b0; b < b1; ++b) {
+            const int L = a.kv_lens[b];
+            a.prefix_out[b] = L - 1;
+            a.suffix_out[b] = 1;
+        }
+    }
     const long long cap = (long long)a.max_pages * a.ps;
     long long sum_s = 0, sum_u = 0;
     bool bad = false;
     for (int b = b0; b < b1; ++b) {
-        const long long P = a.prefix[b], S = a.suffix[b];
-        if (P < 0 || S < 0 || P + S > cap) { bad = true; continue; }
+        const int P = a.prefix[b], S = a.suffix[b];
+        if (P < 0 || S < 0 || (long long)P + S > cap) { bad = true; continue; }
         sum_s += S;
-        sum_u += (long long)a.Hkv * ((S + a.unit_tokens - 1) / a.unit_tokens);
+        sum_u += (long long)a.Hkv * ((S + a.unit_tokens - 1) / a.unit_tokens);  // 32-bit division
     }
     if (bad) s_bad = 1;
+    const bool staged = B <= kSchedSmemAgents;
+    int32_t* s_pre = s_dyn;
+    int32_t* s_suf = s_dyn + B;
+    int32_t* s_uoff = s_dyn + 2 * B;
+    if (staged) {
+        for (int b = b0; b < b1; ++b) {
+            s_pre[b] = a.prefix[b];
+            s_suf[b] = a.suffix[b];
+        }
+    }
     long long inc_s = sum_s, inc_u = sum_u;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -130,13 +164,18 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     const bool ok = !s_bad && tot_s == a.T && tot_s < (1ll << 31) && (!a.build_units || tot_u <= a.max_units);
     if (ok) {
         for (int b = b0; b < b1; ++b) {
-            const long long S = a.suffix[b];
+            const int S = a.suffix[b];
             a.cu[b] = (int32_t)off_s;
             a.unit_off[b] = (int32_t)off_u;
+            if (staged) s_uoff[b] = (int32_t)off_u;
             off_s += S;
             off_u += (long long)a.Hkv * ((S + a.unit_tokens - 1) / a.unit_tokens);
         }
-        if (tid == 0) { a.cu[B] = (int32_t)tot_s; a.unit_off[B] = (int32_t)tot_u; }
+        if (tid == 0) {
+            a.cu[B] = (int32_t)tot_s;
+            a.unit_off[B] = (int32_t)tot_u;
+            if (staged) s_uoff[B] = (int32_t)tot_u;
+        }
     }
     if (!ok) {
         if (tid == 0) {
@@ -149,14 +188,18 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     }
     if (tid == 0) *a.lens_ok = 1;
     if (!a.build_units) return;
+    __syncthreads();  // the staged arrays are complete
+    const int32_t* prefix = staged ? s_pre : a.prefix;
+    const int32_t* suffix = staged ? s_suf : a.suffix;
+    const int32_t* unit_off = staged ? s_uoff : a.unit_off;
 
     // ---- 2. unit costs and their total (the split decision needs it)
     long long my_cost = 0;
     for (long long idx = tid; idx < tot_u; idx += 1024) {
-        const int b = last_le(a.unit_off, B, idx);
-        const int S = a.suffix[b], P = a.prefix[b];
+        const int b = last_le(unit_off, B, idx);
+        const int S = suffix[b], P = prefix[b];
         const int nu = (S + a.unit_tokens - 1) / a.unit_tokens;
-        const int u = (int)(idx - a.unit_off[b]) % nu;
+        const int u = (int)(idx - unit_off[b]) % nu;
         const long long n_keys = (long long)P + min((long long)S, (long long)(u + 1) * a.unit_tokens);
         my_cost += (n_keys + kBN - 1) / kBN;
     }
@@ -170,17 +213,19 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     const long long target = split ? max(8ll, (tot_cost + W * a.split_grid - 1) / (W * a.split_grid)) : 0;
     int my_b = 0, my_g = 0, my_u = 0, my_ns = 1;
     long long my_unit_cost = 0;
+    int my_cost32 = 0;  // the same, in 32 bits (a unit reads fewer than 2^24 tiles: 2^31 keys)
     if (split && tid < tot_u) {  // one unit per thread
-        my_b = last_le(a.unit_off, B, tid);
-        const int S = a.suffix[my_b], P = a.prefix[my_b];
+        my_b = last_le(unit_off, B, tid);
+        const int S = suffix[my_b], P = prefix[my_b];
         const int nu = (S + a.unit_tokens - 1) / a.unit_tokens;
-        const int local = tid - a.unit_off[my_b];
+        const int local = tid - unit_off[my_b];
         my_g = local / nu;
         my_u = local % nu;
         const long long n_keys = (long long)P + min((long long)S, (long long)(my_u + 1) * a.unit_tokens);
         my_unit_cost = (n_keys + kBN - 1) / kBN;
         my_ns = (int)min(min(64ll, my_unit_cost), (my_unit_cost + target - 1) / target);
         if (my_ns < 1) my_ns = 1;
+        my_cost32 = (int)my_unit_cost;
     }
     // partial-result slots and the rank of each split unit (exclusive scans over units)
     long long my_slot_base = 0, my_rank = 0, n_slots = 0, n_split_units = 0;
@@ -192,18 +237,18 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     __syncthreads();
     if (!split) {
         for (long long idx = tid; idx < tot_u; idx += 1024) {
-            const int b = last_le(a.unit_off, B, idx);
-            const int S = a.suffix[b], P = a.prefix[b];
+            const int b = last_le(unit_off, B, idx);
+            const int S = suffix[b], P = prefix[b];
             const int nu = (S + a.unit_tokens - 1) / a.unit_tokens;
-            const int u = (int)(idx - a.unit_off[b]) % nu;
+            const int u = (int)(idx - unit_off[b]) % nu;
             const long long n_keys = (long long)P + min((long long)S, (long long)(u + 1) * a.unit_tokens);
             const long long cost = (n_keys + kBN - 1) / kBN;
             atomicAdd(&s_hist[(int)min(cost, (long long)kCostBuckets - 1)], 1);
         }
     } else if (tid < tot_u) {
         for (int sp = 0; sp < my_ns; ++sp) {
-            const long long c = (sp + 1) * my_unit_cost / my_ns - sp * my_unit_cost / my_ns;
-            atomicAdd(&s_hist[(int)min(c, (long long)kCostBuckets - 1)], 1);
+            const int c = piece_tiles(my_cost32, my_ns, sp);
+            atomicAdd(&s_hist[min(c, kCostBuckets - 1)], 1);
         }
     }
     __syncthreads();
@@ -232,10 +277,10 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     // ---- 5. scatter: item = (agent, kv head | split << 8 | nsplit << 16, unit, KV tiles of the whole unit)
     if (!split) {
         for (long long idx = tid; idx < tot_u; idx += 1024) {
-            const int b = last_le(a.unit_off, B, idx);
-            const int S = a.suffix[b], P = a.prefix[b];
+            const int b = last_le(unit_off, B, idx);
+            const int S = suffix[b], P = prefix[b];
             const int nu = (S + a.unit_tokens - 1) / a.unit_tokens;
-            const int local = (int)(idx - a.unit_off[b]);
+            const int local = (int)(idx - unit_off[b]);
             const int h = local / nu, u = local % nu;
             const long long n_keys = (long long)P + min((long long)S, (long long)(u + 1) * a.unit_tokens);
             const long long cost = (n_keys + kBN - 1) / kBN;
@@ -245,8 +290,8 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
         }
     } else if (tid < tot_u) {
         for (int sp = 0; sp < my_ns; ++sp) {
-            const long long c = (sp + 1) * my_unit_cost / my_ns - sp * my_unit_cost / my_ns;
-            const int pos = atomicAdd(&s_hist[(int)min(c, (long long)kCostBuckets - 1)], 1);
+            const int c = piece_tiles(my_cost32, my_ns, sp);
+            const int pos = atomicAdd(&s_hist[min(c, kCostBuckets - 1)], 1);
             a.units[pos] = make_int4(my_b, my_g | (sp << 8) | (my_ns << 16), my_u, (int)my_unit_cost);
             a.item_slot[pos] = my_ns > 1 ? (int)(my_slot_base + sp) : -1;
         }
@@ -261,7 +306,8 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
 }  // namespace
 
 cudaError_t launch_sched(const SchedArgs& a, cudaStream_t st) {
-    sched_kernel<<<1, 1024, 0, st>>>(a);
+    const size_t smem = a.B <= kSchedSmemAgents ? (size_t)(3 * a.B + 1) * sizeof(int32_t) : 0;
+    sched_kernel<<<1, 1024, smem, st>>>(a);
     return cudaGetLastError();
 }
 
