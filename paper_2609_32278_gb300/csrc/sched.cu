@@ -89,16 +89,10 @@ __device__ void block_exclusive_scan2(long long x, long long y, long long& ex, l
     __syncthreads();
 }
 
-// Batches of at most this many agents keep their lengths and unit offsets in shared memory after the
-// first pass (every later pass, and the binary searches over the unit offsets, would otherwise be
-// chains of dependent global loads); larger batches read them from global memory.
-constexpr int kSchedSmemAgents = 2048;
-
 __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     __shared__ long long s_ws[32], s_wu[32];
     __shared__ int s_hist[kCostBuckets];
     __shared__ int s_bad;
-    extern __shared__ int32_t s_dyn[];  // [prefix: B][suffix: B][unit offsets: B + 1] when staged
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     // the consumer kernel may start its prologue now; it waits for this kernel before reading its output
     ptx::griddep_launch_dependents();
@@ -127,16 +121,6 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
         sum_u += (long long)a.Hkv * ((S + a.unit_tokens - 1) / a.unit_tokens);  // 32-bit division
     }
     if (bad) s_bad = 1;
-    const bool staged = B <= kSchedSmemAgents;
-    int32_t* s_pre = s_dyn;
-    int32_t* s_suf = s_dyn + B;
-    int32_t* s_uoff = s_dyn + 2 * B;
-    if (staged) {
-        for (int b = b0; b < b1; ++b) {
-            s_pre[b] = a.prefix[b];
-            s_suf[b] = a.suffix[b];
-        }
-    }
     long long inc_s = sum_s, inc_u = sum_u;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -167,15 +151,10 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
             const int S = a.suffix[b];
             a.cu[b] = (int32_t)off_s;
             a.unit_off[b] = (int32_t)off_u;
-            if (staged) s_uoff[b] = (int32_t)off_u;
             off_s += S;
             off_u += (long long)a.Hkv * ((S + a.unit_tokens - 1) / a.unit_tokens);
         }
-        if (tid == 0) {
-            a.cu[B] = (int32_t)tot_s;
-            a.unit_off[B] = (int32_t)tot_u;
-            if (staged) s_uoff[B] = (int32_t)tot_u;
-        }
+        if (tid == 0) { a.cu[B] = (int32_t)tot_s; a.unit_off[B] = (int32_t)tot_u; }
     }
     if (!ok) {
         if (tid == 0) {
@@ -188,10 +167,10 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     }
     if (tid == 0) *a.lens_ok = 1;
     if (!a.build_units) return;
-    __syncthreads();  // the staged arrays are complete
-    const int32_t* prefix = staged ? s_pre : a.prefix;
-    const int32_t* suffix = staged ? s_suf : a.suffix;
-    const int32_t* unit_off = staged ? s_uoff : a.unit_off;
+    __syncthreads();  // every thread's cu / unit_off entries are written
+    const int32_t* prefix = a.prefix;
+    const int32_t* suffix = a.suffix;
+    const int32_t* unit_off = a.unit_off;
 
     // ---- 2. unit costs and their total (the split decision needs it)
     long long my_cost = 0;
@@ -306,8 +285,7 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
 }  // namespace
 
 cudaError_t launch_sched(const SchedArgs& a, cudaStream_t st) {
-    const size_t smem = a.B <= kSchedSmemAgents ? (size_t)(3 * a.B + 1) * sizeof(int32_t) : 0;
-    sched_kernel<<<1, 1024, smem, st>>>(a);
+    sched_kernel<<<1, 1024, 0, st>>>(a);
     return cudaGetLastError();
 }
 
