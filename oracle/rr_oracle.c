@@ -31,6 +31,11 @@
  *      are widened to double exactly; everything is computed in double.
  *      `wsum` returns sum_j (w_j / sum_j w_j), which is 1 up to rounding.
  *
+ *  (C) Rotary position embedding of the suffix's q and k rows at positions
+ *      P_b + j (not in the paper; the models its agents run use it -- see
+ *      section (C) below for the reading), and the rounding of a rotated K row
+ *      to the bf16 the pool stores.
+ *
  * Parity of this oracle is pinned in tests/test_oracle_pins.py against a
  * dense brute force with an explicit mask matrix, closed forms and the
  * invariants (prefix-extend equals full causal attention; page permutation
@@ -118,6 +123,7 @@ static void attention_row(const double* qv, const double* K, const double* V, in
 
 typedef struct {
     const uint16_t *q, *k_pool, *v_pool;
+    const double* q64;       /* if set: q as doubles (already rotated by (C)), used instead of q */
     const int32_t *page_table, *prefix_lens, *suffix_lens;
     const int64_t* cu;
     int32_t B, Hq, Hkv, D, ps, max_pages;
@@ -149,8 +155,13 @@ static void paged_item(paged_job* J, int32_t b, int32_t g, double* K, double* V,
         int64_t t = J->cu[b] + i; /* row of q/out */
         for (int32_t hh = 0; hh < G; ++hh) {
             int32_t h = g * G + hh;
-            const uint16_t* qsrc = J->q + (t * J->Hq + h) * (int64_t)D;
-            for (int32_t d = 0; d < D; ++d) qv[d] = widen_bf16(qsrc[d]);
+            if (J->q64) {
+                const double* qsrc = J->q64 + (t * J->Hq + h) * (int64_t)D;
+                for (int32_t d = 0; d < D; ++d) qv[d] = qsrc[d];
+            } else {
+                const uint16_t* qsrc = J->q + (t * J->Hq + h) * (int64_t)D;
+                for (int32_t d = 0; d < D; ++d) qv[d] = widen_bf16(qsrc[d]);
+            }
             int64_t r = t * J->Hq + h;
             attention_row(qv, K, V, P + i, D, J->scale, s, J->out + r * D, J->lse ? J->lse + r : NULL,
                           J->wsum ? J->wsum + r : NULL);
@@ -201,11 +212,11 @@ static int run_threads(void* (*fn)(void*), void* job, int nthreads) {
  * scale <= 0 is NOT replaced here: the caller passes the scale it wants
  * (1/sqrt(D) for the workloads), and scale == 0 is a legal input (uniform weights).
  */
-int oracle_extend_attention(const uint16_t* q, const uint16_t* k_pool, const uint16_t* v_pool,
-                            const int32_t* page_table, const int32_t* prefix_lens, const int32_t* suffix_lens,
-                            int32_t B, int32_t Hq, int32_t Hkv, int32_t D, int32_t ps, int32_t max_pages,
-                            int64_t num_pages, double scale, double* out, double* lse, double* wsum,
-                            int32_t nthreads) {
+static int extend_attention_any(const uint16_t* q, const double* q64, const uint16_t* k_pool,
+                                const uint16_t* v_pool, const int32_t* page_table, const int32_t* prefix_lens,
+                                const int32_t* suffix_lens, int32_t B, int32_t Hq, int32_t Hkv, int32_t D, int32_t ps,
+                                int32_t max_pages, int64_t num_pages, double scale, double* out, double* lse,
+                                double* wsum, int32_t nthreads) {
     if (B < 0 || Hq <= 0 || Hkv <= 0 || Hq % Hkv || D <= 0 || ps <= 0 || max_pages < 0) return ORACLE_BAD_ARG;
     int64_t* cu = (int64_t*)malloc(sizeof(int64_t) * (size_t)(B + 1));
     if (!cu) return ORACLE_NO_MEM;
@@ -220,7 +231,7 @@ int oracle_extend_attention(const uint16_t* q, const uint16_t* k_pool, const uin
     }
     paged_job J;
     memset(&J, 0, sizeof J);
-    J.q = q; J.k_pool = k_pool; J.v_pool = v_pool;
+    J.q = q; J.q64 = q64; J.k_pool = k_pool; J.v_pool = v_pool;
     J.page_table = page_table; J.prefix_lens = prefix_lens; J.suffix_lens = suffix_lens; J.cu = cu;
     J.B = B; J.Hq = Hq; J.Hkv = Hkv; J.D = D; J.ps = ps; J.max_pages = max_pages; J.num_pages = num_pages;
     J.scale = scale; J.out = out; J.lse = lse; J.wsum = wsum;
@@ -231,10 +242,30 @@ int oracle_extend_attention(const uint16_t* q, const uint16_t* k_pool, const uin
     return J.status;
 }
 
+int oracle_extend_attention(const uint16_t* q, const uint16_t* k_pool, const uint16_t* v_pool,
+                            const int32_t* page_table, const int32_t* prefix_lens, const int32_t* suffix_lens,
+                            int32_t B, int32_t Hq, int32_t Hkv, int32_t D, int32_t ps, int32_t max_pages,
+                            int64_t num_pages, double scale, double* out, double* lse, double* wsum,
+                            int32_t nthreads) {
+    return extend_attention_any(q, NULL, k_pool, v_pool, page_table, prefix_lens, suffix_lens, B, Hq, Hkv, D, ps,
+                                max_pages, num_pages, scale, out, lse, wsum, nthreads);
+}
+
+/* The same with q given as doubles [T, Hq, D] (a q rotated by (C) in double precision, not rounded). */
+int oracle_extend_attention_q64(const double* q, const uint16_t* k_pool, const uint16_t* v_pool,
+                                const int32_t* page_table, const int32_t* prefix_lens, const int32_t* suffix_lens,
+                                int32_t B, int32_t Hq, int32_t Hkv, int32_t D, int32_t ps, int32_t max_pages,
+                                int64_t num_pages, double scale, double* out, double* lse, double* wsum,
+                                int32_t nthreads) {
+    return extend_attention_any(NULL, q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, B, Hq, Hkv, D, ps,
+                                max_pages, num_pages, scale, out, lse, wsum, nthreads);
+}
+
 /* ------------------------------- (B) selected rows over one agent's logical K/V */
 
 typedef struct {
     const uint16_t *q, *K, *V;
+    const double* q64;       /* if set: q as doubles, used instead of q */
     const int64_t* positions;
     int64_t n_rows, n_keys;
     int32_t G, D;
@@ -260,8 +291,13 @@ static void* rows_worker(void* arg) {
             if (item >= J->n_rows * J->G) break;
             int64_t r = item / J->G;
             int32_t hh = (int32_t)(item % J->G);
-            const uint16_t* qsrc = J->q + (r * J->G + hh) * (int64_t)J->D;
-            for (int32_t d = 0; d < J->D; ++d) qv[d] = widen_bf16(qsrc[d]);
+            if (J->q64) {
+                const double* qsrc = J->q64 + (r * J->G + hh) * (int64_t)J->D;
+                for (int32_t d = 0; d < J->D; ++d) qv[d] = qsrc[d];
+            } else {
+                const uint16_t* qsrc = J->q + (r * J->G + hh) * (int64_t)J->D;
+                for (int32_t d = 0; d < J->D; ++d) qv[d] = widen_bf16(qsrc[d]);
+            }
             attention_row(qv, J->Kd, J->Vd, J->positions[r], J->D, J->scale, s, J->out + item * J->D,
                           J->lse ? J->lse + item : NULL, J->wsum ? J->wsum + item : NULL);
         }
@@ -277,9 +313,9 @@ static void* rows_worker(void* arg) {
  * row's absolute position (it sees keys 0..positions[r]).
  * out: [n_rows, G, D]; lse, wsum: [n_rows, G] or NULL.
  */
-int oracle_attention_rows(const uint16_t* q, const int64_t* positions, int64_t n_rows, const uint16_t* K,
-                          const uint16_t* V, int64_t n_keys, int32_t G, int32_t D, double scale, double* out,
-                          double* lse, double* wsum, int32_t nthreads) {
+static int attention_rows_any(const uint16_t* q, const double* q64, const int64_t* positions, int64_t n_rows,
+                              const uint16_t* K, const uint16_t* V, int64_t n_keys, int32_t G, int32_t D,
+                              double scale, double* out, double* lse, double* wsum, int32_t nthreads) {
     if (n_rows < 0 || n_keys < 0 || G <= 0 || D <= 0) return ORACLE_BAD_ARG;
     for (int64_t r = 0; r < n_rows; ++r)
         if (positions[r] < 0 || positions[r] >= n_keys) return ORACLE_BAD_ARG;
@@ -295,11 +331,88 @@ int oracle_attention_rows(const uint16_t* q, const int64_t* positions, int64_t n
         J.Kd[e] = widen_bf16(K[e]);
         J.Vd[e] = widen_bf16(V[e]);
     }
-    J.q = q; J.K = K; J.V = V; J.positions = positions; J.n_rows = n_rows; J.n_keys = n_keys;
+    J.q = q; J.q64 = q64; J.K = K; J.V = V; J.positions = positions; J.n_rows = n_rows; J.n_keys = n_keys;
     J.G = G; J.D = D; J.scale = scale; J.out = out; J.lse = lse; J.wsum = wsum;
     pthread_mutex_init(&J.mu, NULL);
     run_threads(rows_worker, &J, nthreads);
     pthread_mutex_destroy(&J.mu);
     free(J.Kd); free(J.Vd);
     return J.status;
+}
+
+int oracle_attention_rows(const uint16_t* q, const int64_t* positions, int64_t n_rows, const uint16_t* K,
+                          const uint16_t* V, int64_t n_keys, int32_t G, int32_t D, double scale, double* out,
+                          double* lse, double* wsum, int32_t nthreads) {
+    return attention_rows_any(q, NULL, positions, n_rows, K, V, n_keys, G, D, scale, out, lse, wsum, nthreads);
+}
+
+/* The same with q_rows given as doubles [n_rows, G, D]. */
+int oracle_attention_rows_q64(const double* q, const int64_t* positions, int64_t n_rows, const uint16_t* K,
+                              const uint16_t* V, int64_t n_keys, int32_t G, int32_t D, double scale, double* out,
+                              double* lse, double* wsum, int32_t nthreads) {
+    return attention_rows_any(NULL, q, positions, n_rows, K, V, n_keys, G, D, scale, out, lse, wsum, nthreads);
+}
+
+/* ------------------------------------------------- (C) rotary position embedding
+ *
+ * The paper never mentions positional encodings.  The models its agents run
+ * (Llama-3, Qwen3) rotate every query and key row by its absolute position
+ * before attention (RoPE: Su et al., "RoFormer: Enhanced Transformer with
+ * Rotary Position Embedding", 2021), so an extend step that receives
+ * un-rotated rows rotates the suffix's q and k at positions P_b + j -- the
+ * positions that continue the cached prefix, which is why the cached keys stay
+ * valid.  Reading used: the "rotate-half" pairing of GPT-NeoX and Llama (dim i
+ * < D/2 pairs with dim i + D/2) and angle p * base^(-2i/D) for pair i:
+ *     y[i]       = x[i]       cos(a) - x[i + D/2] sin(a)
+ *     y[i + D/2] = x[i + D/2] cos(a) + x[i]       sin(a),   a = p * base^(-2i/D)
+ * x: [rows, heads, D] doubles, pos: [rows]; out: [rows, heads, D] doubles.
+ */
+int oracle_rope(const double* x, const int64_t* pos, int64_t rows, int32_t heads, int32_t D, double base,
+                double* out) {
+    if (rows < 0 || heads <= 0 || D <= 0 || D % 2 || !(base > 0.0)) return ORACLE_BAD_ARG;
+    const int32_t half = D / 2;
+    for (int64_t r = 0; r < rows; ++r) {
+        for (int32_t i = 0; i < half; ++i) {
+            const double a = (double)pos[r] * pow(base, -2.0 * i / D);
+            const double c = cos(a), s = sin(a);
+            for (int32_t h = 0; h < heads; ++h) {
+                const double* xr = x + (r * heads + h) * (int64_t)D;
+                double* yr = out + (r * heads + h) * (int64_t)D;
+                yr[i] = xr[i] * c - xr[i + half] * s;
+                yr[i + half] = xr[i + half] * c + xr[i] * s;
+            }
+        }
+    }
+    return ORACLE_OK;
+}
+
+/*
+ * Nearest bfloat16 of each double (8 significant bits, the binary32 exponent
+ * range, subnormals down to 2^-133), ties to even, in ONE rounding from the
+ * double value: the value is scaled so that the bf16 grid around it becomes
+ * the integers, rounded by rint (ties to even in the default rounding mode) and
+ * scaled back.  This is how a bf16 pool stores a K row rotated by (C).
+ */
+int oracle_round_bf16(const double* x, int64_t n, uint16_t* out) {
+    for (int64_t e = 0; e < n; ++e) {
+        double v = x[e];
+        float f;
+        if (isnan(v)) {
+            f = NAN;
+        } else if (v == 0.0 || isinf(v)) {
+            f = (float)v;
+        } else {
+            int ex;
+            frexp(v, &ex);                  /* |v| = m * 2^ex, m in [0.5, 1) */
+            int q = ex - 8;                 /* bf16 spacing in [2^(ex-1), 2^ex) */
+            if (q < -133) q = -133;         /* subnormal spacing */
+            double r = ldexp(rint(ldexp(v, -q)), q);
+            if (fabs(r) >= 0x1.0p128) r = v > 0 ? INFINITY : -INFINITY;
+            f = (float)r;                   /* exact: r is on the bf16 grid */
+        }
+        uint32_t u;
+        memcpy(&u, &f, sizeof u);
+        out[e] = (uint16_t)(u >> 16);
+    }
+    return ORACLE_OK;
 }
