@@ -61,7 +61,7 @@ def kernel_source_hash() -> str:
     """Hash of the attention kernel's code: comments, blank lines and indentation are left out, so an
     edit to the comments keeps a recorded ncu figure valid and any code change invalidates it."""
     h = hashlib.sha256()
-    for f in ("extend_attn.cu", "ptx.cuh", "rr_internal.h"):
+    for f in ("extend_attn.cu", "ptx.cuh", "rope.cuh", "rr_internal.h"):
         with open(os.path.join(ROOT, "paper_2609_32278_gb300", "csrc", f), encoding="utf-8") as fh:
             for line in fh:
                 code = line.split("//", 1)[0].strip()
@@ -559,6 +559,46 @@ def run_ours(args, world, rank, local):
                "overlap": "double-buffered: copies on two side streams overlap the neighbouring steps' kernels"}
         del dev_in, dev_out, out_h, host
 
+    # ---- the same step with rotary position embedding (q and k_new un-rotated; K rotated by the append as
+    # it writes the pool, q by the attention kernel as its tiles land), Llama-3's base 500000
+    rope = None
+    if not args.no_rope:
+        table = rr.rope_table(int((wl.prefix_lens + wl.suffix_lens).max()) + 1, wl.D, 500000.0, device=dev)
+        out_r = torch.empty_like(g["q"])
+
+        def rope_step():
+            rr.kv_append(g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                         g["suffix_lens"], rope=table)
+            rr.extend_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                                g["suffix_lens"], out=out_r, rope=table)
+
+        for _ in range(args.warmup):
+            rope_step()
+        torch.cuda.synchronize(dev)
+        rev = [tuple(torch.cuda.Event(enable_timing=True) for _ in range(3)) for _ in range(args.steps)]
+        for e0, e1, e2 in rev:
+            e0.record(st)
+            rr.kv_append(g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                         g["suffix_lens"], rope=table)
+            e1.record(st)
+            rr.extend_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                                g["suffix_lens"], out=out_r, rope=table)
+            e2.record(st)
+        torch.cuda.synchronize(dev)
+        if rr.device_error():
+            raise RuntimeError("device error in the rotary-step region")
+        r_ms = max_over_ranks(statistics.mean(e0.elapsed_time(e2) for e0, e1, e2 in rev), world, dev)
+        r_app = statistics.mean(e0.elapsed_time(e1) for e0, e1, e2 in rev)
+        r_att = statistics.mean(e1.elapsed_time(e2) for e0, e1, e2 in rev)
+        rope = {"ms_per_step": r_ms, "value": world * F / (r_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
+                "attention_ms": r_att, "attention_tflops": F / (r_att * 1e-3) / 1e12, "kv_append_ms": r_app,
+                "kv_append_gbs": append_bytes(wl) / (r_app * 1e-3) / 1e9, "vs_plain_step": ms_step / r_ms,
+                "base": 500000.0}
+        # restore the un-rotated suffix keys for the legs that follow
+        rr.kv_append(g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                     g["suffix_lens"])
+        del table, out_r
+
     per_agent = None
     if args.per_agent:
         per_agent = per_agent_latency(rr, wl, g, dev, st)
@@ -608,6 +648,8 @@ def run_ours(args, world, rank, local):
         line["per_agent_extend"] = per_agent
     if fused is not None:
         line["fused_step"] = fused
+    if rope is not None:
+        line["rope_step"] = rope
     if decode is not None:
         line["decode"] = decode
     if replay is not None:
@@ -638,6 +680,7 @@ def main():
     ap.add_argument("--decode-config", default="c2_decode", help="decode batch of the decode leg")
     ap.add_argument("--no-decode", action="store_true", help="skip the decode-attention leg")
     ap.add_argument("--no-fused", action="store_true", help="skip the fused extend-step leg")
+    ap.add_argument("--no-rope", action="store_true", help="skip the rotary-embedding step leg")
     ap.add_argument("--decode-agents", type=int, default=0, help="only the first N agents of the decode batch")
     ap.add_argument("--replay", action="store_true",
                     help="also replay synthetic agent traces under each eviction policy (modelled attention TTFT)")

@@ -157,6 +157,76 @@ int rr_decode_attention(const void* q, const void* k_pool, const void* v_pool, c
                         cudaStream_t stream);
 
 /*
+ * Rotary position embedding (RoPE) of the suffix's rows
+ * -----------------------------------------------------
+ * The paper applies no positional encoding of its own, but the models its
+ * agents run (Llama-3, Qwen3) rotate each q and k row by its absolute
+ * position before attention (RoPE: Su et al., "RoFormer", 2021).  The calls
+ * below take the suffix's q and k un-rotated and rotate them at positions
+ * P_b + j -- the positions that continue the cached prefix, which is why the
+ * cached (already rotated) keys stay valid across turns.  Convention: the
+ * "rotate-half" pairing of GPT-NeoX / Llama, dim i < D/2 paired with i + D/2,
+ * pair i at position p turned by a = p * base^(-2i/D):
+ *     y[i] = x[i] cos a - x[i+D/2] sin a,   y[i+D/2] = x[i+D/2] cos a + x[i] sin a
+ * The rotation runs in fp32 from a (cos a, sin a) table and is rounded to
+ * nearest-even bf16: a rotated K row in the pool may differ from the exactly
+ * rounded rotation by one bf16 unit in the last place in rare elements.
+ * Rotating costs no extra pass over HBM: K is rotated by the append as it
+ * writes the pool, q by the attention kernel as each Q tile lands in shared
+ * memory.  Cached prefix keys are read as stored (rotated when they were
+ * appended).
+ */
+
+/*
+ * rr_rope_table -- fill table [max_pos][head_dim/2][2] float (device, 16-byte
+ * aligned, caller-owned) with (cos a, sin a), a = p * base^(-2i/head_dim),
+ * for positions 0 <= p < max_pos and pairs 0 <= i < head_dim/2.  Angles,
+ * cosines and sines are computed in double precision and rounded once to
+ * float.  Build it once per model (base 500000 for Llama-3, 10000 for older
+ * models) with max_pos above the longest context.  head_dim 64 or 128,
+ * base > 1.  Asynchronous on `stream`.
+ */
+int rr_rope_table(float* table, int32_t max_pos, int32_t head_dim, double base, cudaStream_t stream);
+
+/*
+ * rr_kv_append_rope -- rr_kv_append with each K row rotated at its position
+ * P_b + j on its way into the pool (V is copied unchanged).  rope_table /
+ * rope_max_pos: a table built by rr_rope_table for the same head_dim.  A
+ * suffix position >= rope_max_pos is not written and records RR_ERR_LENS in
+ * the device error word.  Other arguments, preconditions and errors as for
+ * rr_kv_append.
+ */
+int rr_kv_append_rope(const void* k_new, const void* v_new, void* k_pool, void* v_pool, const int32_t* page_table,
+                      const int32_t* prefix_lens, const int32_t* suffix_lens, const rr_dims* dims,
+                      const float* rope_table, int32_t rope_max_pos, cudaStream_t stream);
+
+/*
+ * rr_extend_attention_rope -- rr_extend_attention with each suffix query row
+ * rotated at its position P_b + i before its scores are taken (the rotated q
+ * is rounded to bf16 for the tensor cores; q itself is not modified).  The
+ * pool must hold rotated keys (rr_kv_append_rope for the suffix, and the same
+ * for every earlier turn's keys).  A row whose position is >= rope_max_pos is
+ * left un-rotated and records RR_ERR_LENS.  Other arguments as for
+ * rr_extend_attention.
+ */
+int rr_extend_attention_rope(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
+                             const int32_t* prefix_lens, const int32_t* suffix_lens, void* out, const rr_dims* dims,
+                             float softmax_scale, const float* rope_table, int32_t rope_max_pos,
+                             cudaStream_t stream);
+
+/*
+ * rr_extend_step_rope -- the extend step with rotary embedding:
+ * rr_kv_append_rope followed by rr_extend_attention_rope on `stream` (two
+ * launches after their schedules; the one-launch rr_extend_step reads the
+ * suffix keys straight from k_new, which would need rotating in shared memory
+ * on every tile, so it takes rotated rows only).
+ */
+int rr_extend_step_rope(const void* q, const void* k_new, const void* v_new, void* k_pool, void* v_pool,
+                        const int32_t* page_table, const int32_t* prefix_lens, const int32_t* suffix_lens, void* out,
+                        const rr_dims* dims, float softmax_scale, const float* rope_table, int32_t rope_max_pos,
+                        cudaStream_t stream);
+
+/*
  * rr_extend_attention_noalloc -- rr_extend_attention for callers that cannot
  * allocate device memory.  The paper has no counterpart; this is a deployment
  * convenience of this library.

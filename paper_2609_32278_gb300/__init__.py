@@ -7,6 +7,11 @@ suffix):
     kv_append(k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens)
     out = extend_attention(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens)
 
+With rotary position embedding (q and k_new un-rotated; rotated at positions P_b + j):
+
+    rope = rope_table(max_pos, head_dim, base)
+    out = extend_step(q, k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens, rope=rope)
+
 and the step after it, one new token per agent:
 
     kv_append(k_tok, v_tok, k_pool, v_pool, page_table, kv_lens - 1, ones)
@@ -36,7 +41,8 @@ RR_ERR_OVERLAP = 7
 
 # Every symbol include/rr.h declares.
 EXPORTS = ("rr_kv_append", "rr_extend_attention", "rr_extend_step", "rr_decode_attention", "rr_validate_page_table",
-           "rr_get_device_error", "rr_last_error", "rr_version", "rr_shutdown", "rr_extend_attention_noalloc")
+           "rr_get_device_error", "rr_last_error", "rr_version", "rr_shutdown", "rr_extend_attention_noalloc",
+           "rr_rope_table", "rr_kv_append_rope", "rr_extend_attention_rope", "rr_extend_step_rope")
 
 
 class RRError(RuntimeError):
@@ -77,6 +83,15 @@ def lib():
         L.rr_extend_step.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, dp, ctypes.c_float, vp]
         L.rr_decode_attention.restype = ctypes.c_int
         L.rr_decode_attention.argtypes = [vp, vp, vp, vp, vp, vp, dp, ctypes.c_float, vp]
+        L.rr_rope_table.restype = ctypes.c_int
+        L.rr_rope_table.argtypes = [vp, ctypes.c_int32, ctypes.c_int32, ctypes.c_double, vp]
+        L.rr_kv_append_rope.restype = ctypes.c_int
+        L.rr_kv_append_rope.argtypes = [vp, vp, vp, vp, vp, vp, vp, dp, vp, ctypes.c_int32, vp]
+        L.rr_extend_attention_rope.restype = ctypes.c_int
+        L.rr_extend_attention_rope.argtypes = [vp, vp, vp, vp, vp, vp, vp, dp, ctypes.c_float, vp, ctypes.c_int32, vp]
+        L.rr_extend_step_rope.restype = ctypes.c_int
+        L.rr_extend_step_rope.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, dp, ctypes.c_float, vp, ctypes.c_int32,
+                                          vp]
         L.rr_validate_page_table.restype = ctypes.c_int
         L.rr_validate_page_table.argtypes = [vp, vp, vp, dp]
         L.rr_get_device_error.restype = ctypes.c_int
@@ -121,8 +136,29 @@ def make_dims(B, Hq, Hkv, D, ps, max_pages, num_pages, T) -> Dims:
     return Dims(int(B), int(Hq), int(Hkv), int(D), int(ps), int(max_pages), int(num_pages), int(T))
 
 
-def kv_append(k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens, stream=None) -> None:
-    """Write suffix K/V rows into their pool slots (see rr_kv_append in include/rr.h)."""
+def rope_table(max_pos: int, head_dim: int, base: float, device=None, stream=None):
+    """(cos, sin) table of the rotary embedding, float32 [max_pos, head_dim // 2, 2] (rr_rope_table)."""
+    import torch
+    dev = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
+    table = torch.empty((int(max_pos), int(head_dim) // 2, 2), dtype=torch.float32, device=dev)
+    _check(lib().rr_rope_table(table.data_ptr(), int(max_pos), int(head_dim), float(base), _stream_ptr(stream, dev)))
+    return table
+
+
+def _rope_arg(rope, D):
+    """(pointer, max_pos) of a rope_table() tensor, or None."""
+    import torch
+    if rope is None:
+        return None
+    _need(rope, "rope", torch.float32, 3)
+    if rope.shape[1:] != (D // 2, 2):
+        raise ValueError(f"rope table must be [max_pos, {D // 2}, 2] for head dim {D}, got {tuple(rope.shape)}")
+    return rope.data_ptr(), int(rope.shape[0])
+
+
+def kv_append(k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens, stream=None, rope=None) -> None:
+    """Write suffix K/V rows into their pool slots (rr_kv_append); with a rope table, K is rotated at its
+    positions on the way (rr_kv_append_rope)."""
     import torch
     _need(k_new, "k_new", torch.bfloat16, 3)
     _need(v_new, "v_new", torch.bfloat16, 3)
@@ -139,14 +175,19 @@ def kv_append(k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens
     if suffix_lens.shape[0] != B or page_table.shape[0] != B:
         raise ValueError("lens / page_table batch sizes disagree")
     dims = make_dims(B, Hkv, Hkv, D, ps, page_table.shape[1], num_pages, T)
-    _check(lib().rr_kv_append(k_new.data_ptr(), v_new.data_ptr(), k_pool.data_ptr(), v_pool.data_ptr(),
-                              page_table.data_ptr(), prefix_lens.data_ptr(), suffix_lens.data_ptr(),
-                              ctypes.byref(dims), _stream_ptr(stream, k_new.device)))
+    args = (k_new.data_ptr(), v_new.data_ptr(), k_pool.data_ptr(), v_pool.data_ptr(), page_table.data_ptr(),
+            prefix_lens.data_ptr(), suffix_lens.data_ptr(), ctypes.byref(dims))
+    r = _rope_arg(rope, D)
+    if r is None:
+        _check(lib().rr_kv_append(*args, _stream_ptr(stream, k_new.device)))
+    else:
+        _check(lib().rr_kv_append_rope(*args, r[0], r[1], _stream_ptr(stream, k_new.device)))
 
 
 def extend_attention(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, out=None,
-                     softmax_scale: float = 0.0, stream=None):
-    """Extend attention of every suffix row over its agent's prefix + suffix (rr_extend_attention)."""
+                     softmax_scale: float = 0.0, stream=None, rope=None):
+    """Extend attention of every suffix row over its agent's prefix + suffix (rr_extend_attention); with a
+    rope table, each q row is rotated at its position first (rr_extend_attention_rope)."""
     import torch
     _need(q, "q", torch.bfloat16, 3)
     _need(k_pool, "k_pool", torch.bfloat16, 4)
@@ -168,15 +209,20 @@ def extend_attention(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, ou
         if out.shape != q.shape:
             raise ValueError("out must have q's shape")
     dims = make_dims(B, Hq, Hkv, D, ps, page_table.shape[1], num_pages, T)
-    _check(lib().rr_extend_attention(q.data_ptr(), k_pool.data_ptr(), v_pool.data_ptr(), page_table.data_ptr(),
-                                     prefix_lens.data_ptr(), suffix_lens.data_ptr(), out.data_ptr(),
-                                     ctypes.byref(dims), float(softmax_scale), _stream_ptr(stream, q.device)))
+    args = (q.data_ptr(), k_pool.data_ptr(), v_pool.data_ptr(), page_table.data_ptr(), prefix_lens.data_ptr(),
+            suffix_lens.data_ptr(), out.data_ptr(), ctypes.byref(dims), float(softmax_scale))
+    r = _rope_arg(rope, D)
+    if r is None:
+        _check(lib().rr_extend_attention(*args, _stream_ptr(stream, q.device)))
+    else:
+        _check(lib().rr_extend_attention_rope(*args, r[0], r[1], _stream_ptr(stream, q.device)))
     return out
 
 
 def extend_step(q, k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens, out=None,
-                softmax_scale: float = 0.0, stream=None):
-    """kv_append + extend_attention in one attention launch (rr_extend_step): same pools, same output."""
+                softmax_scale: float = 0.0, stream=None, rope=None):
+    """kv_append + extend_attention in one attention launch (rr_extend_step): same pools, same output.
+    With a rope table: the rotated append and the rotated attention (rr_extend_step_rope)."""
     import torch
     _need(q, "q", torch.bfloat16, 3)
     _need(k_new, "k_new", torch.bfloat16, 3)
@@ -200,10 +246,14 @@ def extend_step(q, k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix
         if out.shape != q.shape:
             raise ValueError("out must have q's shape")
     dims = make_dims(B, Hq, Hkv, D, ps, page_table.shape[1], num_pages, T)
-    _check(lib().rr_extend_step(q.data_ptr(), k_new.data_ptr(), v_new.data_ptr(), k_pool.data_ptr(),
-                                v_pool.data_ptr(), page_table.data_ptr(), prefix_lens.data_ptr(),
-                                suffix_lens.data_ptr(), out.data_ptr(), ctypes.byref(dims), float(softmax_scale),
-                                _stream_ptr(stream, q.device)))
+    args = (q.data_ptr(), k_new.data_ptr(), v_new.data_ptr(), k_pool.data_ptr(), v_pool.data_ptr(),
+            page_table.data_ptr(), prefix_lens.data_ptr(), suffix_lens.data_ptr(), out.data_ptr(), ctypes.byref(dims),
+            float(softmax_scale))
+    r = _rope_arg(rope, D)
+    if r is None:
+        _check(lib().rr_extend_step(*args, _stream_ptr(stream, q.device)))
+    else:
+        _check(lib().rr_extend_step_rope(*args, r[0], r[1], _stream_ptr(stream, q.device)))
     return out
 
 

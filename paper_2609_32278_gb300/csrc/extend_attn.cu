@@ -46,6 +46,10 @@
 //   producer loads K(i), V(i) in order; a third V stage keeps it from stalling
 //   on V's stage while K(i+1)'s is already free).
 //
+// Rotary embedding (kRope; rope.cuh): q arrives un-rotated; as a unit's Q tiles land, each softmax
+// thread rotates its own row at position P_b + i in shared memory and arrives on QRot[q], which the
+// MMA issuer waits for before the unit's first S_q.  The keys were rotated by the append.
+//
 // Ordering facts the pipeline relies on: tcgen05.mma operations issued by one
 // thread execute in order, and tcgen05.commit arrives only after every earlier
 // MMA of that thread finished; so when S_q(j) is complete, PV_q(j-1) is too,
@@ -58,6 +62,7 @@
 #include <cuda_bf16.h>
 
 #include "ptx.cuh"
+#include "rope.cuh"
 #include "rr_internal.h"
 
 namespace rr {
@@ -93,7 +98,8 @@ struct Cfg {
     static constexpr int kSFull = 2 + 2 * NK + 2 * NV, kPFull = kSFull + kNQ, kOFinal = kPFull + kNQ;
     static constexpr int kVTmp = kOFinal + kNQ, kDrain = kVTmp + 1, kDone = kDrain + 1;
     static constexpr int kKTmp = kDone + 1;  // fused step: a K tile that needs fixing up before release
-    static constexpr int kNumBars = kKTmp + 1;
+    static constexpr int kQRot = kKTmp + 1;  // rotary q: Q tile q rotated in shared memory (kNQ barriers)
+    static constexpr int kNumBars = kQRot + kNQ;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // u32 TMEM base, i32 abort flag
     static constexpr int kSmemBytes = kOffMisc + 16 + 1024;  // + slack to align the base to 1 KiB
     static_assert(kChunkBytes % 1024 == 0, "swizzle atoms must stay 1 KiB aligned");
@@ -170,10 +176,46 @@ __device__ __forceinline__ int unit_of(int wave, int cta, int grid) {
     return wave * grid + ((wave & 1) ? (grid - 1 - cta) : cta);
 }
 
+// Rotary embedding of one Q row in shared memory (rope.cuh): row r of a Q tile in the 128-byte swizzled
+// layout TMA wrote (16-byte unit u of row r of a 64-column chunk sits at unit u ^ (r & 7)); cs = the
+// (cos, sin) table row of the row's position.  The table and shared-memory loads of four pair units are
+// issued before any of their stores, so a row costs two table round trips, not eight.
+// Not inlined: compiled into the softmax warps' function, this once-per-unit code changed the code of
+// their per-tile loop, and the kernel ran 1.7 % slower with the rotation present but never executed; as
+// a call, the rotating kernel runs at 1.024x the plain one's time on c2 instead of 1.033x.  The rest is
+// the unit boundary: S_q of a unit waits until its Q tile has landed and been rotated.
+template <int D>
+__device__ __noinline__ void rope_q_row(uint8_t* tile, int r, const float2* __restrict__ cs) {
+    auto at = [&](int d) -> uint4* {
+        return reinterpret_cast<uint4*>(tile + (d >> 6) * (kBM * 128) + r * 128 + ((((d & 63) >> 3) ^ (r & 7)) << 4));
+    };
+    constexpr int kUnits = D / 16, kGroup = kUnits < 4 ? kUnits : 4;
+#pragma unroll
+    for (int u0 = 0; u0 < kUnits; u0 += kGroup) {
+        float4 t[kGroup][4];
+        uint4 x0[kGroup], x1[kGroup];
+#pragma unroll
+        for (int k = 0; k < kGroup; ++k) {
+            rope_load8(t[k], cs + 8 * (u0 + k));
+            x0[k] = *at(8 * (u0 + k));
+            x1[k] = *at(8 * (u0 + k) + D / 2);
+        }
+#pragma unroll
+        for (int k = 0; k < kGroup; ++k) {
+            rope_rotate8(x0[k], x1[k], t[k]);
+            *at(8 * (u0 + k)) = x0[k];
+            *at(8 * (u0 + k) + D / 2) = x1[k];
+        }
+    }
+}
+
 // kFused: the one-launch extend step.  Suffix positions' K/V are read from k_new / v_new (the caller's
 // rows, not the pool), and warp 11 writes each work unit's own suffix rows into the pool, so no unit
 // waits for another CTA's pool writes; the attention result is bit-identical to append-then-attend.
-template <int D, int NK, int NV, bool kFused>
+// kRope: q arrives un-rotated; as a unit's Q tiles land, each softmax thread rotates its own row at its
+// position P_b + i in shared memory, and the MMA issuer starts S_q only once tile q is rotated (the
+// keys were rotated on their way into the pool).
+template <int D, int NK, int NV, bool kFused, bool kRope>
 __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_constant__ AttnArgs a) {
     using C = Cfg<D, NK, NV>;
     extern __shared__ uint8_t smem_raw[];
@@ -203,6 +245,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
         }
         ptx::mbar_init(bar(C::kVTmp), 1);
         ptx::mbar_init(bar(C::kKTmp), 1);
+        for (int q = 0; q < kNQ; ++q) ptx::mbar_init(bar(C::kQRot + q), kBM);
         ptx::mbar_init(bar(C::kDrain), 1);
         ptx::mbar_init(bar(C::kDone), 2 * kBM);  // every softmax thread, once, at its end
         *abort_flag = 0;
@@ -479,9 +522,14 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                 {
                     const int sk = (int)(kv_count % NK);
                     if (!(ok = wait_bar(bar(C::kKFull + sk), (kv_count / NK) & 1, ctl))) break;
+                    if (kRope && !(ok = wait_bar(bar(C::kQRot + 0), unit_i & 1, ctl))) break;
                     ptx::tc_fence_after();
                     issue_qk(0, sk);
                     ptx::mma_commit(bar(C::kSFull + 0));
+                    if constexpr (kRope) {
+                        if (!(ok = wait_bar(bar(C::kQRot + 1), unit_i & 1, ctl))) break;
+                        ptx::tc_fence_after();
+                    }
                     issue_qk(1, sk);
                     ptx::mma_commit(bar(C::kSFull + 1));
                     ptx::mma_commit(bar(C::kKEmpty + sk));
@@ -586,7 +634,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
         const uint32_t t_s = tmem + lane_bits + (uint32_t)(q * 128);
         const uint32_t t_o = tmem + lane_bits + 256u + (uint32_t)(q * D);
         const float sl2 = a.scale_log2;
-        uint32_t s_phase = 0, o_phase = 0;
+        uint32_t s_phase = 0, o_phase = 0, q_phase = 0;
         bool ok = true;
         for (int w = 0; ok; ++w) {
             const int ui = unit_of(w, cta, grid);
@@ -598,6 +646,20 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             const int tq0 = u * unit_tokens + q * a.tq;  // first suffix token of this Q tile
             const int row_limit = min(P + tq0 + r / a.G, agent_len - 1);     // last key this row may see
             const int mask_from = (min(P + tq0, agent_len - 1) + 1) / kBN;  // earlier tiles: no masking
+            if constexpr (kRope) {  // rotate this thread's row of Q tile q once the tile has landed
+                if (!(ok = wait_bar(bar(C::kQFull), q_phase, ctl))) break;
+                q_phase ^= 1u;
+                const int tok = tq0 + r / a.G;
+                if (tok < a.suffix[b]) {  // rows past the agent's suffix are never stored
+                    const int pos = P + tok;
+                    if (pos < a.rope_max_pos)
+                        rope_q_row<D>(smem + C::kOffQ + q * C::kQTileBytes, r, a.rope + (long long)pos * (D / 2));
+                    else
+                        atomicCAS(a.err, 0, RR_ERR_LENS);
+                }
+                ptx::fence_proxy_async_smem();  // generic-proxy writes -> the tensor core's reads
+                ptx::mbar_arrive(bar(C::kQRot + q));
+            }
             float m_run = -INFINITY, l_run = 0.f;
             for (int j = kb; j < ke; ++j) {
                 if (!(ok = wait_bar(bar(C::kSFull + q), s_phase, ctl))) break;
@@ -745,7 +807,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
     ptx::mbar_arrive(bar(C::kDone));
 }
 
-template <int D, int NK, int NV, bool kFused>
+template <int D, int NK, int NV, bool kFused, bool kRope>
 cudaError_t launch_cfg(const AttnArgs& a, int grid, cudaStream_t st) {
     using C = Cfg<D, NK, NV>;
     static bool attr_done[64] = {};
@@ -754,12 +816,13 @@ cudaError_t launch_cfg(const AttnArgs& a, int grid, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     if (!attr_done[dev]) {
-        e = cudaFuncSetAttribute(extend_attn_kernel<D, NK, NV, kFused>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(extend_attn_kernel<D, NK, NV, kFused, kRope>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  C::kSmemBytes);
         if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
-    return launch_after_sched(extend_attn_kernel<D, NK, NV, kFused>, dim3(grid), dim3(kThreads), C::kSmemBytes, st, a);
+    return launch_after_sched(extend_attn_kernel<D, NK, NV, kFused, kRope>, dim3(grid), dim3(kThreads), C::kSmemBytes, st,
+                              a);
 }
 
 }  // namespace
@@ -771,8 +834,15 @@ size_t extend_attention_smem_bytes(int head_dim) {
 }
 
 cudaError_t launch_extend_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st, bool fused) {
-    if (head_dim == 128) return fused ? launch_cfg<128, 2, 3, true>(a, grid, st) : launch_cfg<128, 2, 3, false>(a, grid, st);
-    if (head_dim == 64) return fused ? launch_cfg<64, 4, 4, true>(a, grid, st) : launch_cfg<64, 4, 4, false>(a, grid, st);
+    if (fused && a.rope) return cudaErrorInvalidValue;  // the one-launch step takes rotated rows only
+    if (head_dim == 128) {
+        if (fused) return launch_cfg<128, 2, 3, true, false>(a, grid, st);
+        return a.rope ? launch_cfg<128, 2, 3, false, true>(a, grid, st) : launch_cfg<128, 2, 3, false, false>(a, grid, st);
+    }
+    if (head_dim == 64) {
+        if (fused) return launch_cfg<64, 4, 4, true, false>(a, grid, st);
+        return a.rope ? launch_cfg<64, 4, 4, false, true>(a, grid, st) : launch_cfg<64, 4, 4, false, false>(a, grid, st);
+    }
     return cudaErrorInvalidValue;
 }
 

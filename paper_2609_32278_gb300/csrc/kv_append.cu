@@ -12,7 +12,14 @@
 // of traffic, bound by HBM bandwidth.  The suffix rows are read once
 // (streaming loads); the pool writes keep the default policy because the
 // attention kernel reads those pages right after.
+//
+// With a rotary table (kRope), each K row is rotated at its position P_b + j
+// on the way into the pool (rope.cuh): a lane takes the two 16-byte vectors of
+// one head that hold a rotation pair's halves (dims i0.. and i0 + D/2..), so
+// the copy stays one pass over the same bytes plus a table read that the
+// heads of one token share; V is copied unchanged.
 #include "ptx.cuh"
+#include "rope.cuh"
 #include "rr_internal.h"
 
 namespace rr {
@@ -30,6 +37,7 @@ __device__ __forceinline__ int last_le(const int32_t* off, int n, long long x) {
 
 constexpr int kAppendThreads = 256;
 
+template <bool kRope>
 __global__ void __launch_bounds__(kAppendThreads) kv_append_kernel(const AppendArgs a) {
     ptx::griddep_wait();  // the schedule kernel's output (launched as its dependent)
     if (*a.lens_ok == 0) return;
@@ -49,6 +57,32 @@ __global__ void __launch_bounds__(kAppendThreads) kv_append_kernel(const AppendA
         }
         const long long src = t * a.row16;
         const long long dst = ((long long)page * a.ps + pos % a.ps) * a.row16;
+        if constexpr (kRope) {
+            if (pos >= a.rope_max_pos) {  // no table row for this position: nothing written, reported
+                if (lane == 0) atomicCAS(a.err, 0, RR_ERR_LENS);
+                continue;
+            }
+            const float2* cs = a.rope + pos * (long long)(a.d16 * 8);  // this position's D/2 (cos, sin)
+            int e = lane;
+            for (; e + 96 < a.row16; e += 128) {  // V: four vectors in flight per lane, as below
+                uint4 v0 = __ldcs(vn + src + e), v1 = __ldcs(vn + src + e + 32);
+                uint4 v2 = __ldcs(vn + src + e + 64), v3 = __ldcs(vn + src + e + 96);
+                vp[dst + e] = v0; vp[dst + e + 32] = v1; vp[dst + e + 64] = v2; vp[dst + e + 96] = v3;
+            }
+            for (; e < a.row16; e += 32) vp[dst + e] = __ldcs(vn + src + e);
+#pragma unroll 2
+            for (int x = lane; x < a.hkv * a.d16; x += 32) {  // K: the two vectors of one rotation pair unit
+                const int h = x / a.d16, u = x - h * a.d16;
+                const long long lo = (long long)h * 2 * a.d16 + u, hi = lo + a.d16;  // head h: 2 * d16 vectors
+                uint4 k0 = __ldcs(kn + src + lo), k1 = __ldcs(kn + src + hi);
+                float4 t[4];
+                rope_load8(t, cs + u * 8);
+                rope_rotate8(k0, k1, t);
+                kp[dst + lo] = k0;
+                kp[dst + hi] = k1;
+            }
+            continue;
+        }
         int e = lane;
         for (; e + 96 < a.row16; e += 128) {  // four vectors of K and four of V in flight per lane
             uint4 k0 = __ldcs(kn + src + e), k1 = __ldcs(kn + src + e + 32);
@@ -75,7 +109,8 @@ cudaError_t launch_kv_append(const AppendArgs& a, int sm_count, cudaStream_t st)
     const long long cap = (long long)sm_count * 8;  // 8 resident blocks of 256 threads per SM
     if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
-    cudaError_t e = launch_after_sched(kv_append_kernel, dim3((unsigned)blocks), dim3(kAppendThreads), 0, st, a);
+    cudaError_t e = a.rope ? launch_after_sched(kv_append_kernel<true>, dim3((unsigned)blocks), dim3(kAppendThreads), 0, st, a)
+                           : launch_after_sched(kv_append_kernel<false>, dim3((unsigned)blocks), dim3(kAppendThreads), 0, st, a);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }

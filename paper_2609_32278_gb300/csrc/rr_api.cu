@@ -181,12 +181,18 @@ namespace {
 int attention_impl(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
                    const int32_t* prefix_lens, const int32_t* suffix_lens, const int32_t* kv_lens, void* out,
                    const rr_dims* dims, float softmax_scale, cudaStream_t stream, bool decode,
-                   const void* k_new = nullptr, const void* v_new = nullptr) {
+                   const void* k_new = nullptr, const void* v_new = nullptr, const float* rope = nullptr,
+                   int32_t rope_max_pos = 0) {
     g_msg[0] = 0;
     int rc = check_dims(dims, true);
     if (rc) return rc;
     if (dims->total_tokens == 0 && dims->batch == 0) return RR_OK;
     const bool fused = k_new != nullptr || v_new != nullptr;
+    if (rope && dims->total_tokens > 0) {
+        if (!aligned16(rope)) return fail(RR_ERR_INVALID_ARG, "rope table must be 16-byte aligned");
+        if (rope_max_pos <= 0) return fail(RR_ERR_INVALID_ARG, "rope_max_pos must be positive");
+        if (fused || decode) return fail(RR_ERR_UNSUPPORTED, "rotary q is supported by the extend attention call only");
+    }
     if (fused) {
         if (!k_new || !v_new) return fail(RR_ERR_INVALID_ARG, "the fused step needs both k_new and v_new");
         if (!aligned16(k_new) || !aligned16(v_new)) return fail(RR_ERR_INVALID_ARG, "k_new / v_new must be 16-byte aligned");
@@ -309,6 +315,10 @@ int attention_impl(const void* q, const void* k_pool, const void* v_pool, const 
         a.vpool = static_cast<uint4*>(const_cast<void*>(v_pool));
         a.row16 = (int32_t)(row_elems * 2 / 16);
     }
+    if (rope) {
+        a.rope = reinterpret_cast<const float2*>(rope);
+        a.rope_max_pos = rope_max_pos;
+    }
     e = decode ? rr::launch_decode_attention(a, D, (int)std::max<int64_t>(grid, 1), stream)
                : rr::launch_extend_attention(a, D, (int)std::max<int64_t>(grid, 1), stream, fused);
     if (e != cudaSuccess) return cuda_fail(e, decode ? "decode attention kernel launch" : "extend attention kernel launch");
@@ -339,12 +349,21 @@ const char* rr_version(void) { return "rr-extend 0.1 (sm_103a)"; }
 
 const char* rr_last_error(void) { return g_msg; }
 
-int rr_kv_append(const void* k_new, const void* v_new, void* k_pool, void* v_pool, const int32_t* page_table,
-                 const int32_t* prefix_lens, const int32_t* suffix_lens, const rr_dims* dims, cudaStream_t stream) {
+}  // extern "C"
+
+namespace {
+
+int append_impl(const void* k_new, const void* v_new, void* k_pool, void* v_pool, const int32_t* page_table,
+                const int32_t* prefix_lens, const int32_t* suffix_lens, const rr_dims* dims, cudaStream_t stream,
+                const float* rope, int32_t rope_max_pos) {
     g_msg[0] = 0;
     int rc = check_dims(dims, false);
     if (rc) return rc;
     if (dims->total_tokens == 0 && dims->batch == 0) return RR_OK;
+    if (rope && dims->total_tokens > 0) {
+        if (!aligned16(rope)) return fail(RR_ERR_INVALID_ARG, "rope table must be 16-byte aligned");
+        if (rope_max_pos <= 0) return fail(RR_ERR_INVALID_ARG, "rope_max_pos must be positive");
+    }
     if (!page_table || !prefix_lens || !suffix_lens) return fail(RR_ERR_INVALID_ARG, "null lens or page table");
     if (dims->total_tokens > 0 && (!k_new || !v_new || !k_pool || !v_pool))
         return fail(RR_ERR_INVALID_ARG, "null K/V pointer");
@@ -399,9 +418,68 @@ int rr_kv_append(const void* k_new, const void* v_new, void* k_pool, void* v_poo
     a.max_pages = dims->max_pages;
     a.ps = dims->page_size;
     a.row16 = dims->num_kv_heads * dims->head_dim * 2 / 16;
+    if (rope) {
+        a.rope = reinterpret_cast<const float2*>(rope);
+        a.rope_max_pos = rope_max_pos;
+        a.hkv = dims->num_kv_heads;
+        a.d16 = dims->head_dim / 16;
+    }
     e = rr::launch_kv_append(a, d->sm_count, stream);
     if (e != cudaSuccess) return cuda_fail(e, "kv_append kernel launch");
     return RR_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int rr_kv_append(const void* k_new, const void* v_new, void* k_pool, void* v_pool, const int32_t* page_table,
+                 const int32_t* prefix_lens, const int32_t* suffix_lens, const rr_dims* dims, cudaStream_t stream) {
+    return append_impl(k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens, dims, stream, nullptr, 0);
+}
+
+int rr_rope_table(float* table, int32_t max_pos, int32_t head_dim, double base, cudaStream_t stream) {
+    g_msg[0] = 0;
+    if (max_pos < 0) return fail(RR_ERR_INVALID_ARG, "max_pos must be >= 0");
+    if (head_dim != 64 && head_dim != 128) return fail(RR_ERR_UNSUPPORTED, "head_dim %d unsupported (64 or 128)", head_dim);
+    if (!(base > 1.0)) return fail(RR_ERR_INVALID_ARG, "base must be > 1");
+    if (max_pos == 0) return RR_OK;
+    if (!table || !aligned16(table)) return fail(RR_ERR_INVALID_ARG, "table must be a 16-byte aligned device pointer");
+    Device* d = nullptr;
+    int rc = current_device(&d, nullptr);
+    if (rc) return rc;
+    cudaError_t e = rr::launch_rope_table(reinterpret_cast<float2*>(table), max_pos, head_dim, base, d->sm_count, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "rope table kernel launch");
+    return RR_OK;
+}
+
+int rr_kv_append_rope(const void* k_new, const void* v_new, void* k_pool, void* v_pool, const int32_t* page_table,
+                      const int32_t* prefix_lens, const int32_t* suffix_lens, const rr_dims* dims,
+                      const float* rope_table, int32_t rope_max_pos, cudaStream_t stream) {
+    if (!rope_table) return fail(RR_ERR_INVALID_ARG, "null rope table");
+    return append_impl(k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens, dims, stream, rope_table,
+                       rope_max_pos);
+}
+
+int rr_extend_attention_rope(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
+                             const int32_t* prefix_lens, const int32_t* suffix_lens, void* out, const rr_dims* dims,
+                             float softmax_scale, const float* rope_table, int32_t rope_max_pos,
+                             cudaStream_t stream) {
+    if (!rope_table) return fail(RR_ERR_INVALID_ARG, "null rope table");
+    return attention_impl(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, nullptr, out, dims, softmax_scale,
+                          stream, false, nullptr, nullptr, rope_table, rope_max_pos);
+}
+
+int rr_extend_step_rope(const void* q, const void* k_new, const void* v_new, void* k_pool, void* v_pool,
+                        const int32_t* page_table, const int32_t* prefix_lens, const int32_t* suffix_lens, void* out,
+                        const rr_dims* dims, float softmax_scale, const float* rope_table, int32_t rope_max_pos,
+                        cudaStream_t stream) {
+    if (!rope_table) return fail(RR_ERR_INVALID_ARG, "null rope table");
+    int rc = append_impl(k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens, dims, stream, rope_table,
+                         rope_max_pos);
+    if (rc) return rc;
+    return attention_impl(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, nullptr, out, dims, softmax_scale,
+                          stream, false, nullptr, nullptr, rope_table, rope_max_pos);
 }
 
 int rr_extend_attention(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,

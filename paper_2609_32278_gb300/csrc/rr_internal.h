@@ -58,6 +58,10 @@ struct AppendArgs {
     int64_t num_pages;
     int32_t B, max_pages, ps;
     int32_t row16;         // 16-byte vectors per token row (Hkv * D * 2 / 16)
+    // rotary embedding of K (null: plain copy): table [rope_max_pos][D/2] float2 (cos, sin)
+    const float2* rope;
+    int32_t rope_max_pos;
+    int32_t hkv, d16;      // KV heads; D / 16 = rotation pair vectors per head
 };
 
 struct AttnArgs {
@@ -88,6 +92,9 @@ struct AttnArgs {
     uint4* kpool;
     uint4* vpool;
     int32_t row16;         // 16-byte vectors per token row (Hkv * D * 2 / 16)
+    // rotary embedding of q (null: q is used as given): table [rope_max_pos][D/2] float2 (cos, sin)
+    const float2* rope;
+    int32_t rope_max_pos;
 };
 
 struct CombineArgs {
@@ -124,8 +131,11 @@ cudaError_t launch_sched(const SchedArgs& a, cudaStream_t st);
 cudaError_t launch_combine(const CombineArgs& a, int grid, cudaStream_t st);
 cudaError_t launch_kv_append(const AppendArgs& a, int sm_count, cudaStream_t st);
 // Returns cudaErrorInvalidValue for an unsupported head dim.  fused: the one-launch extend step (the
-// suffix K/V come from k_new / v_new, and the kernel also writes them into the pool).
+// suffix K/V come from k_new / v_new, and the kernel also writes them into the pool).  a.rope set: q
+// is rotated in shared memory as each Q tile lands (not with fused).
 cudaError_t launch_extend_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st, bool fused = false);
+// Rotary table (rope.cu): table[p][i] = (cos, sin) of p * base^(-2i/D), p < max_pos, i < D/2.
+cudaError_t launch_rope_table(float2* out, int max_pos, int head_dim, double base, int sm_count, cudaStream_t st);
 size_t extend_attention_smem_bytes(int head_dim);
 // Decode: the same arguments (tm_q boxes one token of G heads); units from the schedule run on
 // prefix = kv_lens - 1 and suffix = 1, which the schedule writes (SchedArgs::kv_lens).

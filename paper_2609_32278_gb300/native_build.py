@@ -10,7 +10,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 OUT = os.path.join(HERE, "librr.so")
 BUILD_DIR = os.path.join(ROOT, "_build")
-SOURCES = ["rr_api.cu", "sched.cu", "kv_append.cu", "extend_attn.cu", "decode_attn.cu", "combine.cu"]
+SOURCES = ["rr_api.cu", "sched.cu", "kv_append.cu", "extend_attn.cu", "decode_attn.cu", "combine.cu", "rope.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
          "-I", os.path.join(ROOT, "include"), "-I", CSRC]
