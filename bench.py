@@ -638,6 +638,8 @@ def run_ours(args, world, rank, local):
                    f"{attn_bytes(wl) / 1e9:.1f} GB > 129 MB)", "parallelism": f"replicas x{world}"},
         "uncached_suffix_tokens_per_s": tok_s,
         "attention_ms": attn_ms, "kv_append_ms": app_ms,
+        "attention_ms_median": statistics.median(ev[k][1].elapsed_time(ev[k][2]) for k in range(args.steps)),
+        "attention_ms_min": min(ev[k][1].elapsed_time(ev[k][2]) for k in range(args.steps)),
         "kv_append_gbs": append_bytes(wl) / (app_ms * 1e-3) / 1e9,
         "roofline": roof,
         "e2e": e2e,
