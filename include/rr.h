@@ -173,8 +173,8 @@ int rr_decode_attention(const void* q, const void* k_pool, const void* v_pool, c
  * rounded rotation by one bf16 unit in the last place in rare elements.
  * Rotating costs no extra pass over HBM: K is rotated by the append as it
  * writes the pool, q by the attention kernel as each Q tile lands in shared
- * memory.  Cached prefix keys are read as stored (rotated when they were
- * appended).
+ * memory (extend and decode alike).  Cached prefix keys are read as stored
+ * (rotated when they were appended).
  */
 
 /*
@@ -225,6 +225,18 @@ int rr_extend_step_rope(const void* q, const void* k_new, const void* v_new, voi
                         const int32_t* page_table, const int32_t* prefix_lens, const int32_t* suffix_lens, void* out,
                         const rr_dims* dims, float softmax_scale, const float* rope_table, int32_t rope_max_pos,
                         cudaStream_t stream);
+
+/*
+ * rr_decode_attention_rope -- rr_decode_attention with each agent's query
+ * rotated at its position L_b - 1 (the new token's) before its scores are
+ * taken; the pool holds rotated keys (the new token's K appended with
+ * rr_kv_append_rope, prefix_lens = L_b - 1, suffix_lens = 1).  A position >=
+ * rope_max_pos leaves that agent's query un-rotated and records RR_ERR_LENS.
+ * Other arguments as for rr_decode_attention.
+ */
+int rr_decode_attention_rope(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
+                             const int32_t* kv_lens, void* out, const rr_dims* dims, float softmax_scale,
+                             const float* rope_table, int32_t rope_max_pos, cudaStream_t stream);
 
 /*
  * rr_extend_attention_noalloc -- rr_extend_attention for callers that cannot

@@ -214,3 +214,13 @@ def extend_attention_rope(q, k_pool, v_pool, page_table, prefix_lens, suffix_len
     return extend_attention(q64, k_pool, v_pool, page_table, prefix_lens, suffix_lens, scale=scale,
                             nthreads=nthreads, with_stats=with_stats)
 
+
+def decode_attention_rope(q, k_pool, v_pool, page_table, kv_lens, base, scale=None, nthreads=0, with_stats=False):
+    """decode_attention with each agent's query rotated at its position kv_lens[b] - 1 (no arithmetic of its
+    own: the lengths are restated and extend_attention_rope computes it)."""
+    L = _c(kv_lens, np.int32)
+    if (L < 1).any():
+        raise OracleError("decode_attention_rope: every agent needs at least its own key")
+    return extend_attention_rope(q, k_pool, v_pool, page_table, L - 1, np.ones_like(L), base, scale=scale,
+                                 nthreads=nthreads, with_stats=with_stats)
+

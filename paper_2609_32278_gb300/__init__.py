@@ -42,7 +42,8 @@ RR_ERR_OVERLAP = 7
 # Every symbol include/rr.h declares.
 EXPORTS = ("rr_kv_append", "rr_extend_attention", "rr_extend_step", "rr_decode_attention", "rr_validate_page_table",
            "rr_get_device_error", "rr_last_error", "rr_version", "rr_shutdown", "rr_extend_attention_noalloc",
-           "rr_rope_table", "rr_kv_append_rope", "rr_extend_attention_rope", "rr_extend_step_rope")
+           "rr_rope_table", "rr_kv_append_rope", "rr_extend_attention_rope", "rr_extend_step_rope",
+           "rr_decode_attention_rope")
 
 
 class RRError(RuntimeError):
@@ -92,6 +93,8 @@ def lib():
         L.rr_extend_step_rope.restype = ctypes.c_int
         L.rr_extend_step_rope.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, dp, ctypes.c_float, vp, ctypes.c_int32,
                                           vp]
+        L.rr_decode_attention_rope.restype = ctypes.c_int
+        L.rr_decode_attention_rope.argtypes = [vp, vp, vp, vp, vp, vp, dp, ctypes.c_float, vp, ctypes.c_int32, vp]
         L.rr_validate_page_table.restype = ctypes.c_int
         L.rr_validate_page_table.argtypes = [vp, vp, vp, dp]
         L.rr_get_device_error.restype = ctypes.c_int
@@ -257,10 +260,12 @@ def extend_step(q, k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix
     return out
 
 
-def decode_attention(q, k_pool, v_pool, page_table, kv_lens, out=None, softmax_scale: float = 0.0, stream=None):
+def decode_attention(q, k_pool, v_pool, page_table, kv_lens, out=None, softmax_scale: float = 0.0, stream=None,
+                     rope=None):
     """Decode attention: the one new query token of each agent over its kv_lens[b] keys (rr_decode_attention).
 
-    q: [B, Hq, D] bf16; kv_lens: [B] int32, the new token's K/V already appended."""
+    q: [B, Hq, D] bf16; kv_lens: [B] int32, the new token's K/V already appended.  With a rope table, q is
+    rotated at position kv_lens[b] - 1 first (rr_decode_attention_rope)."""
     import torch
     _need(q, "q", torch.bfloat16, 3)
     _need(k_pool, "k_pool", torch.bfloat16, 4)
@@ -280,9 +285,13 @@ def decode_attention(q, k_pool, v_pool, page_table, kv_lens, out=None, softmax_s
         if out.shape != q.shape:
             raise ValueError("out must have q's shape")
     dims = make_dims(B, Hq, Hkv, D, ps, page_table.shape[1], num_pages, B)
-    _check(lib().rr_decode_attention(q.data_ptr(), k_pool.data_ptr(), v_pool.data_ptr(), page_table.data_ptr(),
-                                     kv_lens.data_ptr(), out.data_ptr(), ctypes.byref(dims), float(softmax_scale),
-                                     _stream_ptr(stream, q.device)))
+    args = (q.data_ptr(), k_pool.data_ptr(), v_pool.data_ptr(), page_table.data_ptr(), kv_lens.data_ptr(),
+            out.data_ptr(), ctypes.byref(dims), float(softmax_scale))
+    r = _rope_arg(rope, D)
+    if r is None:
+        _check(lib().rr_decode_attention(*args, _stream_ptr(stream, q.device)))
+    else:
+        _check(lib().rr_decode_attention_rope(*args, r[0], r[1], _stream_ptr(stream, q.device)))
     return out
 
 

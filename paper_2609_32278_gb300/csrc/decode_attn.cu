@@ -48,6 +48,7 @@
 #include <cuda_bf16.h>
 
 #include "ptx.cuh"
+#include "rope.cuh"
 #include "rr_internal.h"
 
 namespace rr {
@@ -80,7 +81,8 @@ struct DecCfg {
     static constexpr int kSFull = kVTmp + 1, kSEmpty = kSFull + 2, kPFull = kSEmpty + 2, kPEmpty = kPFull + 2;
     static constexpr int kOFinal = kPEmpty + 2, kOEmpty = kOFinal + 1, kXch = kOEmpty + 1, kDrain = kXch + 1;
     static constexpr int kDone = kDrain + 1;
-    static constexpr int kNumBars = kDone + 1;
+    static constexpr int kQRot = kDone + 1;  // rotary q: the item's Q^T rows rotated in shared memory
+    static constexpr int kNumBars = kQRot + 1;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // u32 TMEM base, i32 abort flag
     static constexpr int kSmemBytes = kOffMisc + 16 + 1024;  // + slack to align the base to 1 KiB
     static_assert(kStageBytes % 1024 == 0 && kOffQ % 1024 == 0 && kOffP % 1024 == 0,
@@ -145,10 +147,38 @@ __device__ __forceinline__ int dec_unit_of(int wave, int cta, int grid) {
     return wave * grid + ((wave & 1) ? (grid - 1 - cta) : cta);
 }
 
+// Rotary embedding of the item's Q^T rows (rope.cuh): the G head rows of the agent's new token, all at
+// position pos = L_b - 1, in the 128-byte swizzled layout TMA wrote (16 rows per 64-column chunk).
+// Softmax thread t takes head row t / (D/16) and rotation pair unit t % (D/16): G * D/16 <= 128 units.
+// Not inlined, to keep the per-tile loop's code as it is without rotation.
+template <int D, int G>
+__device__ __noinline__ void dec_rope_q(uint8_t* qs, int t, const float2* __restrict__ rope, int rope_max_pos, int pos,
+                                        int32_t* err) {
+    constexpr int kUnits = D / 16;
+    const int row = t / kUnits, u = t - row * kUnits;
+    if (row >= G) return;
+    if (pos >= rope_max_pos) {
+        atomicCAS(err, 0, RR_ERR_LENS);
+        return;
+    }
+    auto at = [&](int d) -> uint4* {
+        return reinterpret_cast<uint4*>(qs + (d >> 6) * (kHeadCols * 128) + row * 128 + ((((d & 63) >> 3) ^ (row & 7)) << 4));
+    };
+    uint4* p0 = at(8 * u);
+    uint4* p1 = at(8 * u + D / 2);
+    uint4 x0 = *p0, x1 = *p1;
+    float4 t4[4];
+    rope_load8(t4, rope + (long long)pos * (D / 2) + 8 * u);
+    rope_rotate8(x0, x1, t4);
+    *p0 = x0;
+    *p1 = x1;
+}
+
 // G (query heads per KV head) is a template parameter: every per-head loop below is then unrolled
 // without branches, so the heads' shuffle reductions, shared-memory reads and exponentials
-// interleave instead of running one head after another.
-template <int D, int NS, int G>
+// interleave instead of running one head after another.  kRope: q arrives un-rotated and the softmax
+// warps rotate the item's Q^T rows once they land (dec_rope_q); the MMA thread waits for that.
+template <int D, int NS, int G, bool kRope>
 __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __grid_constant__ AttnArgs a) {
     using C = DecCfg<D, NS>;
     static_assert(G >= 1 && G <= kHeadCols, "one KV head's query heads must fit the 16 MMA columns");
@@ -168,6 +198,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
     if (threadIdx.x == 0) {
         ptx::mbar_init(bar(C::kQFull), 1);
         ptx::mbar_init(bar(C::kQEmpty), 1);
+        ptx::mbar_init(bar(C::kQRot), 128);  // the softmax warps
         for (int s = 0; s < NS; ++s) {
             ptx::mbar_init(bar(C::kKFull + s), 1);
             ptx::mbar_init(bar(C::kVFull + s), 1);
@@ -356,6 +387,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
                 const int sp = (U.y >> 8) & 0xFF, ns = (U.y >> 16) & 0xFF;
                 const int n_kv = (sp + 1) * U.w / ns - sp * U.w / ns;
                 if (!(ok = dec_wait(bar(C::kQFull), item_i & 1, ctl))) break;
+                if (kRope && !(ok = dec_wait(bar(C::kQRot), item_i & 1, ctl))) break;
                 for (int j = 0; j < n_kv && ok; ++j) {
                     const uint32_t t = gt + (uint32_t)j;
                     const int buf = (int)(t & 1);
@@ -406,6 +438,12 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
             const int b = U.x, g = U.y & 0xFF, sp = (U.y >> 8) & 0xFF, ns = (U.y >> 16) & 0xFF;
             const int kb = sp * U.w / ns, ke = (sp + 1) * U.w / ns;
             const int L = a.prefix[b] + 1;
+            if constexpr (kRope) {  // rotate the item's Q^T rows once they have landed
+                if (!(ok = dec_wait(bar(C::kQFull), item_i & 1, ctl))) break;
+                dec_rope_q<D, G>(smem + C::kOffQ, threadIdx.x, a.rope, a.rope_max_pos, L - 1, a.err);
+                ptx::fence_proxy_async_smem();  // generic-proxy writes -> the tensor core's reads
+                ptx::mbar_arrive(bar(C::kQRot));
+            }
             float m[G], lp[G];
 #pragma unroll
             for (int h = 0; h < G; ++h) { m[h] = -INFINITY; lp[h] = 0.f; }
@@ -550,7 +588,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
     ptx::mbar_arrive(bar(C::kDone));
 }
 
-template <int D, int NS, int G>
+template <int D, int NS, int G, bool kRope>
 cudaError_t launch_dec(const AttnArgs& a, int grid, cudaStream_t st) {
     using C = DecCfg<D, NS>;
     static bool attr_done[64] = {};
@@ -559,22 +597,23 @@ cudaError_t launch_dec(const AttnArgs& a, int grid, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     if (!attr_done[dev]) {
-        e = cudaFuncSetAttribute(decode_attn_kernel<D, NS, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(decode_attn_kernel<D, NS, G, kRope>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  C::kSmemBytes);
         if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
-    return launch_after_sched(decode_attn_kernel<D, NS, G>, dim3(grid), dim3(kDecThreads), C::kSmemBytes, st, a);
+    return launch_after_sched(decode_attn_kernel<D, NS, G, kRope>, dim3(grid), dim3(kDecThreads), C::kSmemBytes, st,
+                              a);
 }
 
-template <int D, int NS>
+template <int D, int NS, bool kRope>
 cudaError_t launch_dec_g(const AttnArgs& a, int grid, cudaStream_t st) {
     switch (a.G) {
-        case 1: return launch_dec<D, NS, 1>(a, grid, st);
-        case 2: return launch_dec<D, NS, 2>(a, grid, st);
-        case 4: return launch_dec<D, NS, 4>(a, grid, st);
-        case 8: return launch_dec<D, NS, 8>(a, grid, st);
-        case 16: return launch_dec<D, NS, 16>(a, grid, st);
+        case 1: return launch_dec<D, NS, 1, kRope>(a, grid, st);
+        case 2: return launch_dec<D, NS, 2, kRope>(a, grid, st);
+        case 4: return launch_dec<D, NS, 4, kRope>(a, grid, st);
+        case 8: return launch_dec<D, NS, 8, kRope>(a, grid, st);
+        case 16: return launch_dec<D, NS, 16, kRope>(a, grid, st);
         default: return cudaErrorInvalidValue;
     }
 }
@@ -582,8 +621,8 @@ cudaError_t launch_dec_g(const AttnArgs& a, int grid, cudaStream_t st) {
 }  // namespace
 
 cudaError_t launch_decode_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st) {
-    if (head_dim == 128) return launch_dec_g<128, 3>(a, grid, st);
-    if (head_dim == 64) return launch_dec_g<64, 6>(a, grid, st);
+    if (head_dim == 128) return a.rope ? launch_dec_g<128, 3, true>(a, grid, st) : launch_dec_g<128, 3, false>(a, grid, st);
+    if (head_dim == 64) return a.rope ? launch_dec_g<64, 6, true>(a, grid, st) : launch_dec_g<64, 6, false>(a, grid, st);
     return cudaErrorInvalidValue;
 }
 

@@ -191,7 +191,7 @@ int attention_impl(const void* q, const void* k_pool, const void* v_pool, const 
     if (rope && dims->total_tokens > 0) {
         if (!aligned16(rope)) return fail(RR_ERR_INVALID_ARG, "rope table must be 16-byte aligned");
         if (rope_max_pos <= 0) return fail(RR_ERR_INVALID_ARG, "rope_max_pos must be positive");
-        if (fused || decode) return fail(RR_ERR_UNSUPPORTED, "rotary q is supported by the extend attention call only");
+        if (fused) return fail(RR_ERR_UNSUPPORTED, "the one-launch extend step takes rotated rows only");
     }
     if (fused) {
         if (!k_new || !v_new) return fail(RR_ERR_INVALID_ARG, "the fused step needs both k_new and v_new");
@@ -494,6 +494,14 @@ int rr_decode_attention(const void* q, const void* k_pool, const void* v_pool, c
                         cudaStream_t stream) {
     return attention_impl(q, k_pool, v_pool, page_table, nullptr, nullptr, kv_lens, out, dims, softmax_scale, stream,
                           true);
+}
+
+int rr_decode_attention_rope(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
+                             const int32_t* kv_lens, void* out, const rr_dims* dims, float softmax_scale,
+                             const float* rope_table, int32_t rope_max_pos, cudaStream_t stream) {
+    if (!rope_table) return fail(RR_ERR_INVALID_ARG, "null rope table");
+    return attention_impl(q, k_pool, v_pool, page_table, nullptr, nullptr, kv_lens, out, dims, softmax_scale, stream,
+                          true, nullptr, nullptr, rope_table, rope_max_pos);
 }
 
 int rr_extend_step(const void* q, const void* k_new, const void* v_new, void* k_pool, void* v_pool,

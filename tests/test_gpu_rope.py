@@ -1,5 +1,5 @@
 """Rotary position embedding on the GPU (rr_rope_table, rr_kv_append_rope, rr_extend_attention_rope,
-rr_extend_step_rope) against the fp64 oracle, on the same seeded inputs.
+rr_extend_step_rope, rr_decode_attention_rope) against the fp64 oracle, on the same seeded inputs.
 
 * the (cos, sin) table against the oracle's rotation of unit vectors (float rounding of the double
   values);
@@ -10,7 +10,9 @@ rr_extend_step_rope) against the fp64 oracle, on the same seeded inputs.
   not rounded; the oracle's own rotated pool): every GQA group, both head dims, prefixes in the middle of
   a page, split-K batches, positions past 10^5 (angles the table must hold to float accuracy);
 * the one-call step bit-identical to its two calls; a position past the table reported, and the library
-  usable afterwards.
+  usable afterwards;
+* decode with rotary embedding (q rotated at L_b - 1 by the decode kernel) within the parity bar of the
+  oracle: every GQA group, both head dims, split-K, positions past 10^5.
 """
 import math
 
@@ -204,4 +206,53 @@ def test_rope_position_past_table_is_reported(rr):
     table = rr.rope_table(200, 128, BASE)
     g = synth.gpu_tensors(wl, "cuda")
     out = _run_gpu_rope(rr, wl, g, table)
+    assert torch.isfinite(out.float()).all()
+
+
+DECODE_CASES = [
+    # name, B, Hq, Hkv, D, kv_lens
+    ("dec_d128_g4", 4, 8, 2, 128, [300, 1000, 129, 2048]),
+    ("dec_d128_g16", 2, 16, 1, 128, [900, 260]),
+    ("dec_d64_g8", 2, 16, 2, 64, [555, 4096]),
+    ("dec_d128_g1", 2, 2, 2, 128, [640, 33]),
+    ("dec_d64_g2", 3, 4, 2, 64, [1, 17, 300]),
+    ("dec_split_long", 1, 8, 2, 128, [20000]),
+    ("dec_positions_past_1e5", 1, 8, 2, 128, [150001]),
+]
+
+
+@pytest.mark.parametrize("case", DECODE_CASES, ids=[c[0] for c in DECODE_CASES])
+def test_rope_decode_against_oracle(rr, case):
+    """Decode with rotary embedding: the new token's K rotated by the append, its q by the decode kernel."""
+    import torch
+    name, B, Hq, Hkv, D, L = case
+    L = np.asarray(L, dtype=np.int64)
+    wl = synth.custom(name, B, Hq, Hkv, D, L - 1, np.ones(B, dtype=np.int64), seed=19)
+    host = synth.cpu_tensors(wl)
+    g = synth.gpu_tensors(wl, "cuda")
+    table = rr.rope_table(int(L.max()), D, BASE)
+    rr.kv_append(g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                 g["suffix_lens"], rope=table)
+    kv_lens = (g["prefix_lens"] + 1).to(torch.int32)
+    out = rr.decode_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"], kv_lens, rope=table)
+    assert rr.device_error() == 0, rr.last_error()
+    kp, vp = oracle.kv_append_rope(host["k_new"], host["v_new"], host["k_pool"], host["v_pool"], wl.page_table,
+                                   wl.prefix_lens, wl.suffix_lens, BASE)
+    ref = oracle.decode_attention_rope(host["q"], kp, vp, wl.page_table, L, BASE, scale=1.0 / math.sqrt(D))
+    check_close(to_f64(out), ref, name)
+
+
+def test_rope_decode_position_past_table_is_reported(rr):
+    import torch
+    wl = synth.custom("dec_short_table", 2, 8, 2, 128, [99, 10], [1, 1], seed=20)
+    g = synth.gpu_tensors(wl, "cuda")
+    table = rr.rope_table(200, 128, BASE)
+    rr.kv_append(g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                 g["suffix_lens"], rope=table)
+    assert rr.device_error() == 0
+    kv_lens = (g["prefix_lens"] + 1).to(torch.int32)
+    rr.decode_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"], kv_lens, rope=rr.rope_table(50, 128, BASE))
+    assert rr.device_error() == rr.RR_ERR_LENS      # agent 0's token sits at position 99
+    out = rr.decode_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"], kv_lens, rope=table)
+    assert rr.device_error() == 0
     assert torch.isfinite(out.float()).all()
