@@ -22,12 +22,25 @@ def to_f64(t) -> np.ndarray:
     return synth.bf16_to_f64(bf16_bits(t))
 
 
+def _ordered(bits: np.ndarray) -> np.ndarray:
+    """bf16 bit patterns -> integers in the order of their values (one step = one unit in the last place)."""
+    b = bits.astype(np.int64)
+    return np.where(b & 0x8000, -(b & 0x7FFF), b)
+
+
 def check_close(got: np.ndarray, ref: np.ndarray, what: str = "") -> dict:
+    """Parity of a bf16 GPU output (as float64) with the fp64 oracle: max and mean |err| against the bar,
+    plus the 99.9th percentile |err| and the distance in bf16 units in the last place to the oracle
+    rounded to bf16 (round to nearest even, once), printed on one line."""
     err = np.abs(got - ref)
     stats = dict(n=int(err.size), max=float(err.max()) if err.size else 0.0,
                  mean=float(err.mean()) if err.size else 0.0,
                  p999=float(np.quantile(err, 0.999)) if err.size else 0.0)
     assert np.isfinite(got).all(), f"{what}: non-finite outputs"
+    if err.size:
+        ulp = np.abs(_ordered(oracle.round_bf16(got)) - _ordered(oracle.round_bf16(ref)))
+        stats.update(ulp_max=int(ulp.max()), ulp_le1=float(np.mean(ulp <= 1)), ulp_eq0=float(np.mean(ulp == 0)))
+    print(f"parity {what}: {stats}")
     assert stats["max"] <= MAX_ABS and stats["mean"] <= MEAN_ABS, f"{what}: {stats}"
     return stats
 
