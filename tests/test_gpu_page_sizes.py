@@ -1,4 +1,5 @@
-"""Every supported page size (8, 16, 32, 64, 128 tokens): append, extend, decode and the fused step.
+"""Every supported page size (8, 16, 32, 64, 128 tokens): append, extend, decode, the fused step and the
+rotary-embedding calls.
 
 The page gather issues one TMA box per page (128 / page_size lanes per 128-key tile), the append
 and the fused writer index slots by position % page_size, and the last-page clearing depends on
@@ -102,3 +103,37 @@ def test_split_k(rr, ps):
     assert rr.device_error() == 0, rr.last_error()
     _, _, ref = oracle_step(wl)
     check_close(to_f64(out), ref, f"split ps={ps}")
+
+
+@pytest.mark.parametrize("ps", PAGE_SIZES)
+def test_rotary_extend_and_decode(rr, ps):
+    """Rotary embedding at every page size: the rotated append indexes slots by position % page_size."""
+    import torch
+    base = 500000.0
+    wl = synth.custom(f"rope_ps{ps}", 3, 8, 2, 128, [37, 300, 0], [129, 70, 200], ps=ps, seed=4)
+    h = synth.cpu_tensors(wl)
+    g = synth.gpu_tensors(wl, "cuda")
+    table = rr.rope_table(600, 128, base)
+    out = rr.extend_step(g["q"], g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"],
+                         g["prefix_lens"], g["suffix_lens"], rope=table)
+    assert rr.device_error() == 0, rr.last_error()
+    kp, vp = oracle.kv_append_rope(h["k_new"], h["v_new"], h["k_pool"], h["v_pool"], wl.page_table,
+                                   wl.prefix_lens, wl.suffix_lens, base)
+    np.testing.assert_array_equal(u16(g["v_pool"]), vp)
+    ref = oracle.extend_attention_rope(h["q"], kp, vp, wl.page_table, wl.prefix_lens, wl.suffix_lens, base,
+                                       scale=1.0 / math.sqrt(wl.D))
+    check_close(to_f64(out), ref, f"rotary extend ps={ps}")
+    # decode over one new token per agent at its next position
+    L = np.array([400, 77, 513], dtype=np.int64)
+    wd = synth.custom(f"rope_dec_ps{ps}", 3, 8, 2, 128, L - 1, np.ones(3, dtype=np.int64), ps=ps, seed=5)
+    hd = synth.cpu_tensors(wd)
+    gd = synth.gpu_tensors(wd, "cuda")
+    rr.kv_append(gd["k_new"], gd["v_new"], gd["k_pool"], gd["v_pool"], gd["page_table"], gd["prefix_lens"],
+                 gd["suffix_lens"], rope=table)
+    kv = (gd["prefix_lens"] + 1).to(torch.int32)
+    outd = rr.decode_attention(gd["q"], gd["k_pool"], gd["v_pool"], gd["page_table"], kv, rope=table)
+    assert rr.device_error() == 0, rr.last_error()
+    kpd, vpd = oracle.kv_append_rope(hd["k_new"], hd["v_new"], hd["k_pool"], hd["v_pool"], wd.page_table,
+                                     wd.prefix_lens, wd.suffix_lens, base)
+    refd = oracle.decode_attention_rope(hd["q"], kpd, vpd, wd.page_table, L, base, scale=1.0 / math.sqrt(wd.D))
+    check_close(to_f64(outd), refd, f"rotary decode ps={ps}")
