@@ -15,6 +15,7 @@
 // nsplit * (D + 2) floats per row, writes D bf16.
 #include <cuda_bf16.h>
 
+#include "ptx.cuh"
 #include "rr_internal.h"
 
 namespace rr {
@@ -27,6 +28,7 @@ template <int D>
 __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const CombineArgs a) {
     static_assert(D == 64 || D == 128, "lane mapping: 2 or 4 columns per lane");
     constexpr int kPer = D / 32;  // columns per lane
+    ptx::griddep_wait();  // launched as the attention kernel's dependent: its partials must be complete
     const int n = *a.n_split;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int unit_tokens = kNQ * a.tq;
@@ -86,9 +88,11 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const CombineA
 
 cudaError_t launch_combine(const CombineArgs& a, int grid, cudaStream_t st) {
     if (grid < 1) grid = 1;
-    if (a.D == 128) combine_kernel<128><<<grid, kCombineThreads, 0, st>>>(a);
-    else if (a.D == 64) combine_kernel<64><<<grid, kCombineThreads, 0, st>>>(a);
+    cudaError_t e;
+    if (a.D == 128) e = launch_after_sched(combine_kernel<128>, dim3(grid), dim3(kCombineThreads), 0, st, a);
+    else if (a.D == 64) e = launch_after_sched(combine_kernel<64>, dim3(grid), dim3(kCombineThreads), 0, st, a);
     else return cudaErrorInvalidValue;
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 

@@ -108,9 +108,10 @@ struct CombineArgs {
     int32_t Hq, G, D, tq;
 };
 
-// Launch `kernel` so that it may start while the schedule kernel before it on the stream finishes
-// (programmatic dependent launch); the kernel must call ptx::griddep_wait() before it reads anything
-// the schedule writes.
+// Launch `kernel` so that it may start while the kernel before it on the stream finishes (programmatic
+// dependent launch: the schedule before the append and attention kernels, the attention kernel before
+// the split-K combine); the kernel must call ptx::griddep_wait() before it reads anything the kernels
+// before it write.
 template <typename... KArgs, typename... Args>
 cudaError_t launch_after_sched(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
                                Args&&... args) {
