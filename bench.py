@@ -323,6 +323,30 @@ def decode_leg(args, rr, synth, dev, st, peaks, rank):
                         "kernel": f"decode_attn_kernel<{wl.D},{3 if wl.D == 128 else 6},{wl.G}>",
                         "peak_kind": f"{peaks['src']} HBM copy bandwidth"},
            "l2": f"K/V working set {nbytes / 1e9:.1f} GB > 129 MB"}
+    # a batch over a common prefix: the same calls through rr_decode_attention_shared (the shared pages read
+    # once per group of 16 / G agents), checked against the plain call's output within the parity bar
+    if wl.shared_len > 0 and wl.shared_len % 128 == 0 and wl.B * wl.Hkv <= 1024:
+        out_s = torch.empty_like(out)
+        for _ in range(max(3, args.warmup)):
+            rr.decode_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"], kv_lens, out=out_s,
+                                shared_len=wl.shared_len)
+        torch.cuda.synchronize(dev)
+        for e0, e1 in ev:
+            e0.record(st)
+            rr.decode_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"], kv_lens, out=out_s,
+                                shared_len=wl.shared_len)
+            e1.record(st)
+        torch.cuda.synchronize(dev)
+        if rr.device_error():
+            raise RuntimeError("device error in the shared-prefix decode region")
+        diff = (out_s.float() - out.float()).abs()
+        if float(diff.max()) > 2e-2:
+            raise RuntimeError("shared-prefix decode differs from the plain decode")
+        ms_s = statistics.mean(e0.elapsed_time(e1) for e0, e1 in ev)
+        res["shared_prefix"] = {"shared_len": int(wl.shared_len), "ms_per_call": ms_s,
+                                "tokens_per_s": wl.B / (ms_s * 1e-3), "vs_plain": ms / ms_s,
+                                "algorithmic_gbs_of_plain_bytes": nbytes / (ms_s * 1e-3) / 1e9}
+        del out_s
     del g, out, kv_lens
     torch.cuda.empty_cache()
     return res

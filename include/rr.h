@@ -56,6 +56,7 @@ extern "C" {
 #define RR_ERR_OOB 5           /* device or host: a page id outside [0, num_pages) */
 #define RR_ERR_LENS 6          /* device: negative length, P_b+S_b > max_pages*ps, or sum S_b != T */
 #define RR_ERR_OVERLAP 7       /* host validation: a suffix page is shared with another agent or a prefix */
+#define RR_ERR_SHARED 8        /* device: an agent's page table differs from agent 0's inside the declared shared prefix */
 
 /* Sizes of one call.  All counts are in elements or tokens, not bytes. */
 typedef struct rr_dims {
@@ -225,6 +226,30 @@ int rr_extend_step_rope(const void* q, const void* k_new, const void* v_new, voi
                         const int32_t* page_table, const int32_t* prefix_lens, const int32_t* suffix_lens, void* out,
                         const rr_dims* dims, float softmax_scale, const float* rope_table, int32_t rope_max_pos,
                         cudaStream_t stream);
+
+/*
+ * rr_decode_attention_shared -- rr_decode_attention for a batch whose agents
+ * all share their first shared_len positions (a common system prompt, the
+ * same physical pages at the start of every page table: Sec. 2's shared
+ * prefix cache).  Same result as rr_decode_attention (within the parity
+ * tolerance: the merge order differs), fewer bytes: the shared pages are read
+ * once per group of 16 / G agents of a KV head -- their queries fill the 16
+ * columns the tensor-core MMA has, which G query heads alone leave mostly
+ * padding -- instead of once per agent; each agent's keys from shared_len on
+ * are read as by rr_decode_attention, and the two partial results of every
+ * (agent, query head) are merged by their log-sum-exp weights.
+ *
+ * shared_len: a positive multiple of 128 with shared_len < kv_lens[b] for
+ * every agent (each agent's own new token lies past the shared prefix).  The
+ * device records RR_ERR_LENS if an agent's kv_lens is not larger, and
+ * RR_ERR_SHARED if an agent's first shared_len / page_size page-table entries
+ * differ from agent 0's.  Batches of more than 1024 (agent, KV head) pairs are
+ * computed by rr_decode_attention.  Other arguments, layouts and errors as for
+ * rr_decode_attention.
+ */
+int rr_decode_attention_shared(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
+                               const int32_t* kv_lens, int32_t shared_len, void* out, const rr_dims* dims,
+                               float softmax_scale, cudaStream_t stream);
 
 /*
  * rr_decode_attention_rope -- rr_decode_attention with each agent's query

@@ -38,12 +38,13 @@ RR_ERR_TIMEOUT = 4
 RR_ERR_OOB = 5
 RR_ERR_LENS = 6
 RR_ERR_OVERLAP = 7
+RR_ERR_SHARED = 8
 
 # Every symbol include/rr.h declares.
 EXPORTS = ("rr_kv_append", "rr_extend_attention", "rr_extend_step", "rr_decode_attention", "rr_validate_page_table",
            "rr_get_device_error", "rr_last_error", "rr_version", "rr_shutdown", "rr_extend_attention_noalloc",
            "rr_rope_table", "rr_kv_append_rope", "rr_extend_attention_rope", "rr_extend_step_rope",
-           "rr_decode_attention_rope")
+           "rr_decode_attention_rope", "rr_decode_attention_shared")
 
 
 class RRError(RuntimeError):
@@ -93,6 +94,8 @@ def lib():
         L.rr_extend_step_rope.restype = ctypes.c_int
         L.rr_extend_step_rope.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, dp, ctypes.c_float, vp, ctypes.c_int32,
                                           vp]
+        L.rr_decode_attention_shared.restype = ctypes.c_int
+        L.rr_decode_attention_shared.argtypes = [vp, vp, vp, vp, vp, ctypes.c_int32, vp, dp, ctypes.c_float, vp]
         L.rr_decode_attention_rope.restype = ctypes.c_int
         L.rr_decode_attention_rope.argtypes = [vp, vp, vp, vp, vp, vp, dp, ctypes.c_float, vp, ctypes.c_int32, vp]
         L.rr_validate_page_table.restype = ctypes.c_int
@@ -261,11 +264,12 @@ def extend_step(q, k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix
 
 
 def decode_attention(q, k_pool, v_pool, page_table, kv_lens, out=None, softmax_scale: float = 0.0, stream=None,
-                     rope=None):
+                     rope=None, shared_len: int = 0):
     """Decode attention: the one new query token of each agent over its kv_lens[b] keys (rr_decode_attention).
 
     q: [B, Hq, D] bf16; kv_lens: [B] int32, the new token's K/V already appended.  With a rope table, q is
-    rotated at position kv_lens[b] - 1 first (rr_decode_attention_rope)."""
+    rotated at position kv_lens[b] - 1 first (rr_decode_attention_rope).  shared_len > 0: every agent's first
+    shared_len positions are the same pages, read once per group of agents (rr_decode_attention_shared)."""
     import torch
     _need(q, "q", torch.bfloat16, 3)
     _need(k_pool, "k_pool", torch.bfloat16, 4)
@@ -288,7 +292,14 @@ def decode_attention(q, k_pool, v_pool, page_table, kv_lens, out=None, softmax_s
     args = (q.data_ptr(), k_pool.data_ptr(), v_pool.data_ptr(), page_table.data_ptr(), kv_lens.data_ptr(),
             out.data_ptr(), ctypes.byref(dims), float(softmax_scale))
     r = _rope_arg(rope, D)
-    if r is None:
+    if shared_len:
+        if r is not None:
+            raise ValueError("the shared-prefix decode takes rotated queries only")
+        _check(lib().rr_decode_attention_shared(q.data_ptr(), k_pool.data_ptr(), v_pool.data_ptr(),
+                                                page_table.data_ptr(), kv_lens.data_ptr(), int(shared_len),
+                                                out.data_ptr(), ctypes.byref(dims), float(softmax_scale),
+                                                _stream_ptr(stream, q.device)))
+    elif r is None:
         _check(lib().rr_decode_attention(*args, _stream_ptr(stream, q.device)))
     else:
         _check(lib().rr_decode_attention_rope(*args, r[0], r[1], _stream_ptr(stream, q.device)))

@@ -10,8 +10,9 @@
 // first piece always holds key 0, so M is finite.  The pieces are merged in a
 // fixed order, so the result is deterministic.
 //
-// One block per split unit (256 rows: two Q tiles of 128 packed rows); a warp
-// takes a row at a time, each lane 4 of the D columns.  Memory bound: reads
+// One block per split unit (a.rows partial rows per piece: two Q tiles of 128
+// packed rows for extend, one row per query head for decode); a warp takes a
+// row at a time, each lane 4 of the D columns.  Memory bound: reads
 // nsplit * (D + 2) floats per row, writes D bf16.
 #include <cuda_bf16.h>
 
@@ -36,7 +37,7 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const CombineA
         const int4 su = a.split_units[k];
         const int b = su.x, g = su.y & 0xFF, ns = (su.y >> 16) & 0xFF, u = su.z, base = su.w;
         const int S = a.suffix[b], cu_b = a.cu[b];
-        for (int row = warp; row < kNQ * kBM; row += kCombineThreads / 32) {
+        for (int row = warp; row < a.rows; row += kCombineThreads / 32) {
             const int q = row / kBM, rr = row % kBM;
             const int tok = u * unit_tokens + q * a.tq + rr / a.G;
             if (tok >= S) continue;
@@ -45,13 +46,13 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const CombineA
             // is a chain of dependent global loads otherwise: ~2 x nsplit memory latencies per row).
             float M = -INFINITY;
 #pragma unroll 8
-            for (int s = 0; s < ns; ++s) M = fmaxf(M, a.part_ml[(long long)(base + s) * (kNQ * kBM) + row].x);
+            for (int s = 0; s < ns; ++s) M = fmaxf(M, a.part_ml[(long long)(base + s) * a.rows + row].x);
             float L = 0.f, acc[kPer];
 #pragma unroll
             for (int i = 0; i < kPer; ++i) acc[i] = 0.f;
 #pragma unroll 4
             for (int s = 0; s < ns; ++s) {
-                const long long prow = (long long)(base + s) * (kNQ * kBM) + row;
+                const long long prow = (long long)(base + s) * a.rows + row;
                 const float2 ml = a.part_ml[prow];
                 const float w = ml.x == -INFINITY ? 0.f : exp2f(ml.x - M);
                 L += w * ml.y;

@@ -174,13 +174,51 @@ __device__ __noinline__ void dec_rope_q(uint8_t* qs, int t, const float2* __rest
     *p1 = x1;
 }
 
+// One work item: agent b (the first of the group for a shared-prefix item), KV head g, piece sp, its KV
+// tiles [kb, ke) counted from the first tile the item's range starts at, and the number of keys L of that
+// range (its last key is L - 1).
+struct DecItem {
+    int b, g, sp, kb, ke, L;
+};
+
+template <bool kGroup>
+__device__ __forceinline__ DecItem dec_item(const AttnArgs& a, int ui) {
+    DecItem it;
+    if constexpr (kGroup) {
+        // shared-prefix item ui = ((g * groups_per_head) + group) * group_ns + piece
+        const int ns = a.group_ns;
+        it.sp = ui % ns;
+        const int t = ui / ns;
+        it.g = t / a.groups_per_head;
+        it.b = (t % a.groups_per_head) * a.group_agents;
+        it.kb = it.sp * a.shared_tiles / ns;
+        it.ke = (it.sp + 1) * a.shared_tiles / ns;
+        it.L = a.shared_tiles * kBN;
+    } else {
+        const int4 U = a.units[ui];
+        it.b = U.x;
+        it.g = U.y & 0xFF;
+        it.sp = (U.y >> 8) & 0xFF;
+        const int ns = (U.y >> 16) & 0xFF;
+        it.kb = it.sp * U.w / ns;
+        it.ke = (it.sp + 1) * U.w / ns;
+        it.L = a.prefix[it.b] + 1;  // keys of the agent (its private keys over a shared prefix), the new token's included
+    }
+    return it;
+}
+
 // G (query heads per KV head) is a template parameter: every per-head loop below is then unrolled
 // without branches, so the heads' shuffle reductions, shared-memory reads and exponentials
 // interleave instead of running one head after another.  kRope: q arrives un-rotated and the softmax
 // warps rotate the item's Q^T rows once they land (dec_rope_q); the MMA thread waits for that.
-template <int D, int NS, int G, bool kRope>
+//
+// kGroup: the shared-prefix items of rr_decode_attention_shared.  G is then 16, the MMA's columns: the
+// a.G query heads of a.group_agents consecutive agents (Q^T loaded through tm_qg), all over the same
+// shared pages; each column's partial result goes to its agent's unit slot.
+template <int D, int NS, int G, bool kRope, bool kGroup = false>
 __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __grid_constant__ AttnArgs a) {
     using C = DecCfg<D, NS>;
+    static_assert(!(kRope && kGroup), "shared-prefix items take rotated queries only");
     static_assert(G >= 1 && G <= kHeadCols, "one KV head's query heads must fit the 16 MMA columns");
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -233,8 +271,11 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
     ptx::tc_fence_after();
     const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + C::kOffMisc);
     ptx::griddep_wait();  // the schedule kernel's output (launched as its dependent)
-    const int n_units = *a.n_units;
+    // shared-prefix items: as many as the host set up, but none if the schedule rejected the batch (it then
+    // lists no private items and has written no unit slots)
+    const int n_units = kGroup ? (*a.n_units > 0 ? a.group_items : 0) : *a.n_units;
     const int grid = gridDim.x, cta = blockIdx.x;
+    const int page0 = kGroup ? 0 : a.page0;  // page-table column of the item range's first key
 
     if (warp == kDecWarpProducer) {
         // ------------------------------------------------------------ TMA producer
@@ -246,18 +287,23 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
         for (int w = 0; ok; ++w) {
             const int ui = dec_unit_of(w, cta, grid);
             if (ui >= n_units) break;
-            const int4 U = a.units[ui];
-            const int b = U.x, g = U.y & 0xFF, sp = (U.y >> 8) & 0xFF, ns = (U.y >> 16) & 0xFF;
-            const int kb = sp * U.w / ns, ke = (sp + 1) * U.w / ns;
-            const int L = a.prefix[b] + 1;  // keys of the agent, the new token included
+            const DecItem it = dec_item<kGroup>(a, ui);
+            const int b = it.b, g = it.g, kb = it.kb, ke = it.ke, L = it.L;
             const int last_page_end = ((L + a.ps - 1) / a.ps) * a.ps;
             if (lane == 0) {
                 if (item_i > 0) ok = dec_wait(bar(C::kQEmpty), (item_i - 1) & 1, ctl);
                 if (ok) {
+                    // one box of 16 Q^T rows (group: group_agents agents x a.G heads; rows past the batch are
+                    // zero-filled) or G rows, per 64-column chunk
                     ptx::mbar_arrive_expect_tx(bar(C::kQFull), C::kChunks * G * 128);
-                    for (int c = 0; c < C::kChunks; ++c)
-                        ptx::tma_load_3d(sb + C::kOffQ + c * C::kNarrowChunkBytes, &a.tm_q, c * 64, g * G, a.cu[b],
-                                         bar(C::kQFull));
+                    for (int c = 0; c < C::kChunks; ++c) {
+                        if constexpr (kGroup)
+                            ptx::tma_load_3d(sb + C::kOffQ + c * C::kNarrowChunkBytes, &a.tm_qg, c * 64, g * a.G, b,
+                                             bar(C::kQFull));
+                        else
+                            ptx::tma_load_3d(sb + C::kOffQ + c * C::kNarrowChunkBytes, &a.tm_q, c * 64, g * G, a.cu[b],
+                                             bar(C::kQFull));
+                    }
                     armed_q = (int)(item_i & 1);
                 }
             }
@@ -270,7 +316,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
                 if (lane < ppt) {
                     const int lp = j * ppt + lane;
                     if (lp * a.ps < L) {
-                        const int pid = a.page_table[(long long)b * a.max_pages + lp];
+                        const int pid = a.page_table[(long long)b * a.max_pages + page0 + lp];
                         if (pid >= 0 && (long long)pid < a.num_pages) row = pid * a.ps;
                         else atomicCAS(a.err, 0, RR_ERR_OOB);
                     }
@@ -383,9 +429,8 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
             for (int w = 0; ok; ++w) {
                 const int ui = dec_unit_of(w, cta, grid);
                 if (ui >= n_units) break;
-                const int4 U = a.units[ui];
-                const int sp = (U.y >> 8) & 0xFF, ns = (U.y >> 16) & 0xFF;
-                const int n_kv = (sp + 1) * U.w / ns - sp * U.w / ns;
+                const DecItem it = dec_item<kGroup>(a, ui);
+                const int n_kv = it.ke - it.kb;
                 if (!(ok = dec_wait(bar(C::kQFull), item_i & 1, ctl))) break;
                 if (kRope && !(ok = dec_wait(bar(C::kQRot), item_i & 1, ctl))) break;
                 for (int j = 0; j < n_kv && ok; ++j) {
@@ -434,10 +479,8 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
         for (int w = 0; ok; ++w) {
             const int ui = dec_unit_of(w, cta, grid);
             if (ui >= n_units) break;
-            const int4 U = a.units[ui];
-            const int b = U.x, g = U.y & 0xFF, sp = (U.y >> 8) & 0xFF, ns = (U.y >> 16) & 0xFF;
-            const int kb = sp * U.w / ns, ke = (sp + 1) * U.w / ns;
-            const int L = a.prefix[b] + 1;
+            const DecItem it = dec_item<kGroup>(a, ui);
+            const int b = it.b, g = it.g, kb = it.kb, ke = it.ke, L = it.L;
             if constexpr (kRope) {  // rotate the item's Q^T rows once they have landed
                 if (!(ok = dec_wait(bar(C::kQFull), item_i & 1, ctl))) break;
                 dec_rope_q<D, G>(smem + C::kOffQ, threadIdx.x, a.rope, a.rope_max_pos, L - 1, a.err);
@@ -564,14 +607,24 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
             tmem_wait_ld16(o);
             ptx::tc_fence_before();
             ptx::mbar_arrive(bar(C::kOEmpty));
-            const int slot = a.item_slot[ui];
+            const int slot = kGroup ? 0 : a.item_slot[ui];
             if (t_in < D) {
 #pragma unroll
                 for (int h = 0; h < G; ++h) {
                     const float lsum = (rx[h] + rx[kHeadCols + h]) + (rx[2 * kHeadCols + h] + rx[3 * kHeadCols + h]);
-                    if (slot >= 0) {
+                    if constexpr (kGroup) {
+                        // column h: query head h % a.G of agent b + h / a.G; its piece sp of the shared prefix goes to
+                        // slot sp of the agent's unit (the unit's private pieces follow)
+                        const int ag = b + h / a.G;
+                        if (h / a.G < a.group_agents && ag < a.batch) {
+                            const int us = a.unit_slot[(long long)ag * (a.Hq / a.G) + g] + it.sp;
+                            const long long prow = (long long)us * a.rows_per_slot + h % a.G;
+                            a.part_o[prow * D + t_in] = __uint_as_float(o[h]);
+                            if (t_in == 0) a.part_ml[prow] = make_float2(m[h], lsum);
+                        }
+                    } else if (slot >= 0) {
                         // split item: fp32 unnormalised O row h of the unit plus (max, sum)
-                        const long long prow = (long long)slot * (kNQ * kBM) + h;
+                        const long long prow = (long long)slot * a.rows_per_slot + h;
                         a.part_o[prow * D + t_in] = __uint_as_float(o[h]);
                         if (t_in == 0) a.part_ml[prow] = make_float2(m[h], lsum);
                     } else {
@@ -588,7 +641,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
     ptx::mbar_arrive(bar(C::kDone));
 }
 
-template <int D, int NS, int G, bool kRope>
+template <int D, int NS, int G, bool kRope, bool kGroup = false>
 cudaError_t launch_dec(const AttnArgs& a, int grid, cudaStream_t st) {
     using C = DecCfg<D, NS>;
     static bool attr_done[64] = {};
@@ -597,13 +650,13 @@ cudaError_t launch_dec(const AttnArgs& a, int grid, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     if (!attr_done[dev]) {
-        e = cudaFuncSetAttribute(decode_attn_kernel<D, NS, G, kRope>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(decode_attn_kernel<D, NS, G, kRope, kGroup>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  C::kSmemBytes);
         if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
-    return launch_after_sched(decode_attn_kernel<D, NS, G, kRope>, dim3(grid), dim3(kDecThreads), C::kSmemBytes, st,
-                              a);
+    return launch_after_sched(decode_attn_kernel<D, NS, G, kRope, kGroup>, dim3(grid), dim3(kDecThreads), C::kSmemBytes,
+                              st, a);
 }
 
 template <int D, int NS, bool kRope>
@@ -623,6 +676,13 @@ cudaError_t launch_dec_g(const AttnArgs& a, int grid, cudaStream_t st) {
 cudaError_t launch_decode_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st) {
     if (head_dim == 128) return a.rope ? launch_dec_g<128, 3, true>(a, grid, st) : launch_dec_g<128, 3, false>(a, grid, st);
     if (head_dim == 64) return a.rope ? launch_dec_g<64, 6, true>(a, grid, st) : launch_dec_g<64, 6, false>(a, grid, st);
+    return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_decode_shared_prefix(const AttnArgs& a, int head_dim, int grid, cudaStream_t st) {
+    if (a.rope || a.group_agents * a.G != kHeadCols) return cudaErrorInvalidValue;
+    if (head_dim == 128) return launch_dec<128, 3, kHeadCols, false, true>(a, grid, st);
+    if (head_dim == 64) return launch_dec<64, 6, kHeadCols, false, true>(a, grid, st);
     return cudaErrorInvalidValue;
 }
 

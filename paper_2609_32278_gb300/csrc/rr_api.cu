@@ -48,11 +48,13 @@ size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 // [item_slot: max_items][split units: max_split x int4][part_ml: slots x 256 float2][part_o: slots x 256 x D]
 // [decode only: prefix B][suffix B]
 struct Layout {
-    size_t off_cu, off_unit_off, off_units, off_slot, off_split, off_ml, off_o, off_lens, total;
+    size_t off_cu, off_unit_off, off_units, off_slot, off_split, off_ml, off_o, off_lens, off_uslot, total;
 };
 
+// rows: partial rows per slot (two Q tiles for extend, 16 for decode); unit_slots: entries of the decode
+// shared-prefix call's first-slot-per-unit array.
 Layout layout_for(int64_t B, int64_t max_items, int64_t max_split = 0, int64_t slots = 0, int64_t D = 0,
-                  bool lens = false) {
+                  bool lens = false, int64_t rows = rr::kNQ * rr::kBM, int64_t unit_slots = 0) {
     Layout L;
     L.off_cu = 256;
     L.off_unit_off = L.off_cu + align256((size_t)(B + 1) * 4);
@@ -60,9 +62,10 @@ Layout layout_for(int64_t B, int64_t max_items, int64_t max_split = 0, int64_t s
     L.off_slot = L.off_units + align256((size_t)max_items * 16);
     L.off_split = L.off_slot + align256((size_t)max_items * 4);
     L.off_ml = L.off_split + align256((size_t)max_split * 16);
-    L.off_o = L.off_ml + align256((size_t)slots * rr::kNQ * rr::kBM * 8);
-    L.off_lens = L.off_o + align256((size_t)slots * rr::kNQ * rr::kBM * (size_t)D * 4);
-    L.total = L.off_lens + (lens ? 2 * align256((size_t)B * 4) : 0);  // decode: prefix, suffix arrays
+    L.off_o = L.off_ml + align256((size_t)slots * rows * 8);
+    L.off_lens = L.off_o + align256((size_t)slots * rows * (size_t)D * 4);
+    L.off_uslot = L.off_lens + (lens ? 2 * align256((size_t)B * 4) : 0);  // decode: prefix, suffix arrays
+    L.total = L.off_uslot + align256((size_t)unit_slots * 4);
     return L;
 }
 
@@ -234,7 +237,8 @@ int attention_impl(const void* q, const void* k_pool, const void* v_pool, const 
     const int64_t max_split = may_split ? 2ll * grid_sm : 0;
     const int64_t slots = may_split ? (int64_t)(split_waves + 2) * grid_sm : 0;
     const int64_t max_items = std::max<int64_t>(max_units, slots);
-    const Layout L = layout_for(B, max_items, max_split, slots, D, decode);
+    const int64_t rows_per_slot = decode ? 16 : rr::kNQ * rr::kBM;
+    const Layout L = layout_for(B, max_items, max_split, slots, D, decode, rows_per_slot);
     if ((rc = ensure_ws(*d, L.total))) return rc;
     uint8_t* ws = static_cast<uint8_t*>(d->ws);
     cudaError_t e = cudaSuccess;
@@ -291,6 +295,7 @@ int attention_impl(const void* q, const void* k_pool, const void* v_pool, const 
     a.n_units = s.n_units;
     a.item_slot = s.item_slot;
     a.part_o = reinterpret_cast<float*>(ws + L.off_o);
+    a.rows_per_slot = (int32_t)rows_per_slot;
     a.part_ml = reinterpret_cast<float2*>(ws + L.off_ml);
     a.err = d->err;
     a.out = out;
@@ -335,9 +340,165 @@ int attention_impl(const void* q, const void* k_pool, const void* v_pool, const 
         c.G = G;
         c.D = D;
         c.tq = tq;
+        c.rows = (int32_t)rows_per_slot;
         e = rr::launch_combine(c, (int)max_split, stream);
         if (e != cudaSuccess) return cuda_fail(e, "split-K combine kernel launch");
     }
+    return RR_OK;
+}
+
+// Decode over a prefix every agent of the batch shares (rr_decode_attention_shared): the shared prefix's
+// pages are read once per group of 16 / G agents (their queries fill the MMA's 16 columns) instead of once
+// per agent, each agent's private keys by the plain decode kernel, and both partial results are merged.
+int decode_shared_impl(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
+                       const int32_t* kv_lens, int32_t shared_len, void* out, const rr_dims* dims,
+                       float softmax_scale, cudaStream_t stream) {
+    g_msg[0] = 0;
+    int rc = check_dims(dims, true);
+    if (rc) return rc;
+    if (dims->batch == 0) return RR_OK;
+    if (!page_table || !kv_lens) return fail(RR_ERR_INVALID_ARG, "null kv_lens or page table");
+    if (dims->total_tokens != dims->batch)
+        return fail(RR_ERR_INVALID_ARG, "decode takes one query token per agent: total_tokens (%lld) != batch (%d)",
+                    (long long)dims->total_tokens, dims->batch);
+    if (!q || !k_pool || !v_pool || !out) return fail(RR_ERR_INVALID_ARG, "null q/pool/out pointer");
+    if (!aligned16(q) || !aligned16(k_pool) || !aligned16(v_pool) || !aligned16(out))
+        return fail(RR_ERR_INVALID_ARG, "q, pools and out must be 16-byte aligned");
+    if (!aligned4(page_table) || !aligned4(kv_lens)) return fail(RR_ERR_INVALID_ARG, "int32 arrays must be 4-byte aligned");
+    if (dims->num_pages == 0) return fail(RR_ERR_INVALID_ARG, "empty pool");
+    const int Hq = dims->num_q_heads, Hkv = dims->num_kv_heads, D = dims->head_dim, ps = dims->page_size;
+    const int G = Hq / Hkv;
+    const int64_t B = dims->batch;
+    if (shared_len <= 0 || shared_len % rr::kBN != 0)
+        return fail(RR_ERR_UNSUPPORTED, "shared_len (%d) must be a positive multiple of %d", shared_len, rr::kBN);
+    if ((int64_t)shared_len > (int64_t)dims->max_pages * ps) return fail(RR_ERR_INVALID_ARG, "shared_len exceeds max_pages");
+    // the schedule gives each thread of one block one (agent, KV head) unit: larger batches take the plain call
+    if (B * Hkv > 1024)
+        return attention_impl(q, k_pool, v_pool, page_table, nullptr, nullptr, kv_lens, out, dims, softmax_scale, stream,
+                              true);
+
+    Device* d = nullptr;
+    if ((rc = current_device(&d, nullptr))) return rc;
+    if ((rc = get_encoder())) return rc;
+    const int grid_sm = d->sm_count;
+    const int tq = rr::kBM / G;
+    const int unit_tokens = rr::kNQ * tq;
+    const int64_t units = B * Hkv;
+    // shared-prefix items: one KV head x group_agents agents x one of group_ns pieces of the shared tiles;
+    // enough pieces for two waves
+    const int group_agents = 16 / G;
+    const int64_t groups_per_head = (B + group_agents - 1) / group_agents;
+    const int shared_tiles = shared_len / rr::kBN;
+    const int64_t groups = groups_per_head * Hkv;
+    const int group_ns = (int)std::max<int64_t>(
+        1, std::min<int64_t>(std::min(64, shared_tiles), (2ll * grid_sm + groups - 1) / groups));
+    const int split_waves = 6;
+    // slots: every unit's group_ns shared pieces plus its private pieces (1 each, or a split into at most
+    // (waves + 2) x grid pieces over all units)
+    const int64_t slots = units * group_ns + std::max<int64_t>(units, (int64_t)(split_waves + 2) * grid_sm);
+    const int64_t max_items = std::max<int64_t>(units, (int64_t)(split_waves + 2) * grid_sm);
+    const Layout L = layout_for(B, max_items, units, slots, D, true, 16, units);
+    if ((rc = ensure_ws(*d, L.total))) return rc;
+    uint8_t* ws = static_cast<uint8_t*>(d->ws);
+    int32_t* prefix_lens = reinterpret_cast<int32_t*>(ws + L.off_lens);
+    int32_t* suffix_lens = reinterpret_cast<int32_t*>(ws + L.off_lens + align256((size_t)B * 4));
+    int32_t* unit_slot = reinterpret_cast<int32_t*>(ws + L.off_uslot);
+
+    rr::SchedArgs s{};
+    s.kv_lens = kv_lens;
+    s.prefix_out = prefix_lens;
+    s.suffix_out = suffix_lens;
+    s.prefix = prefix_lens;
+    s.suffix = suffix_lens;
+    s.lens_offset = shared_len;
+    s.extra_slots = group_ns;
+    s.unit_slot = unit_slot;
+    s.page_table = page_table;
+    s.shared_pages = shared_len / ps;
+    s.B = (int32_t)B;
+    s.Hkv = Hkv;
+    s.unit_tokens = unit_tokens;
+    s.T = B;
+    s.max_pages = dims->max_pages;
+    s.ps = ps;
+    s.max_units = units;
+    s.build_units = 1;
+    s.cu = reinterpret_cast<int32_t*>(ws + L.off_cu);
+    s.unit_off = reinterpret_cast<int32_t*>(ws + L.off_unit_off);
+    s.units = reinterpret_cast<int4*>(ws + L.off_units);
+    s.item_slot = reinterpret_cast<int32_t*>(ws + L.off_slot);
+    s.split_units = reinterpret_cast<int4*>(ws + L.off_split);
+    s.n_split = reinterpret_cast<int32_t*>(ws) + 2;
+    s.split_grid = grid_sm;
+    s.split_waves = split_waves;
+    s.n_units = reinterpret_cast<int32_t*>(ws);
+    s.lens_ok = reinterpret_cast<int32_t*>(ws) + 1;
+    s.err = d->err;
+    cudaError_t e = rr::launch_sched(s, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "schedule kernel launch");
+
+    rr::AttnArgs a;
+    memset(&a, 0, sizeof a);
+    if ((rc = encode_3d(&a.tm_q, q, (uint64_t)D, (uint64_t)Hq, (uint64_t)B, (uint64_t)D * 2, (uint64_t)Hq * D * 2, 64,
+                        (uint32_t)G, 1u)))
+        return rc;
+    if ((rc = encode_3d(&a.tm_qg, q, (uint64_t)D, (uint64_t)Hq, (uint64_t)B, (uint64_t)D * 2, (uint64_t)Hq * D * 2, 64,
+                        (uint32_t)G, (uint32_t)group_agents)))
+        return rc;
+    const uint64_t rows = (uint64_t)dims->num_pages * (uint64_t)ps;
+    if ((rc = encode_2d(&a.tm_k, k_pool, (uint64_t)Hkv * D, rows, (uint64_t)Hkv * D * 2, 64, (uint32_t)ps))) return rc;
+    if ((rc = encode_2d(&a.tm_v, v_pool, (uint64_t)Hkv * D, rows, (uint64_t)Hkv * D * 2, 64, (uint32_t)ps))) return rc;
+    a.page_table = page_table;
+    a.prefix = prefix_lens;
+    a.suffix = suffix_lens;
+    a.cu = s.cu;
+    a.units = s.units;
+    a.n_units = s.n_units;
+    a.item_slot = s.item_slot;
+    a.part_o = reinterpret_cast<float*>(ws + L.off_o);
+    a.part_ml = reinterpret_cast<float2*>(ws + L.off_ml);
+    a.rows_per_slot = 16;
+    a.err = d->err;
+    a.out = out;
+    a.num_pages = dims->num_pages;
+    a.Hq = Hq;
+    a.G = G;
+    a.ps = ps;
+    a.max_pages = dims->max_pages;
+    a.tq = tq;
+    a.oob_row = (int32_t)rows;
+    const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)D);
+    a.scale_log2 = scale * 1.4426950408889634f;
+    a.unit_slot = unit_slot;
+    a.batch = (int32_t)B;
+    // 1. the shared prefix, once per group of agents
+    a.group_items = (int32_t)(groups * group_ns);
+    a.group_ns = group_ns;
+    a.group_agents = group_agents;
+    a.groups_per_head = (int32_t)groups_per_head;
+    a.shared_tiles = shared_tiles;
+    e = rr::launch_decode_shared_prefix(a, D, (int)std::min<int64_t>(grid_sm, groups * group_ns), stream);
+    if (e != cudaSuccess) return cuda_fail(e, "shared-prefix decode kernel launch");
+    // 2. every agent's private keys, from page-table column shared_len / ps on
+    a.page0 = shared_len / ps;
+    e = rr::launch_decode_attention(a, D, (int)std::min<int64_t>(grid_sm, max_items), stream);
+    if (e != cudaSuccess) return cuda_fail(e, "decode attention kernel launch");
+    // 3. merge each (agent, query head)'s shared and private pieces
+    rr::CombineArgs c;
+    c.split_units = s.split_units;
+    c.n_split = s.n_split;
+    c.part_o = a.part_o;
+    c.part_ml = a.part_ml;
+    c.suffix = suffix_lens;
+    c.cu = s.cu;
+    c.out = out;
+    c.Hq = Hq;
+    c.G = G;
+    c.D = D;
+    c.tq = tq;
+    c.rows = 16;
+    e = rr::launch_combine(c, (int)std::min<int64_t>(units, 2ll * grid_sm), stream);
+    if (e != cudaSuccess) return cuda_fail(e, "split-K combine kernel launch");
     return RR_OK;
 }
 
@@ -494,6 +655,12 @@ int rr_decode_attention(const void* q, const void* k_pool, const void* v_pool, c
                         cudaStream_t stream) {
     return attention_impl(q, k_pool, v_pool, page_table, nullptr, nullptr, kv_lens, out, dims, softmax_scale, stream,
                           true);
+}
+
+int rr_decode_attention_shared(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
+                               const int32_t* kv_lens, int32_t shared_len, void* out, const rr_dims* dims,
+                               float softmax_scale, cudaStream_t stream) {
+    return decode_shared_impl(q, k_pool, v_pool, page_table, kv_lens, shared_len, out, dims, softmax_scale, stream);
 }
 
 int rr_decode_attention_rope(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,

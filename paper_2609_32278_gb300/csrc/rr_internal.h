@@ -39,6 +39,15 @@ struct SchedArgs {
     int32_t* n_split;      // number of split units
     int32_t split_grid;    // persistent grid size; 0 disables splitting
     int32_t split_waves;   // a split aims at this many waves of items (2 if 0); slots needed: (waves + 2) x grid
+    // decode over a shared prefix (rr_decode_attention_shared): the schedule covers each agent's private keys
+    // (kv_lens - lens_offset of them); every unit writes partial results, into slots after `extra_slots`
+    // slots reserved for the shared prefix's pieces; unit_slot[b * Hkv + g] receives the unit's first slot.
+    // shared_pages > 0: every agent's first shared_pages page-table entries must equal agent 0's.
+    int32_t lens_offset;
+    int32_t extra_slots;
+    int32_t* unit_slot;
+    const int32_t* page_table;
+    int32_t shared_pages;
     int32_t* n_units;      // number of items
     int32_t* lens_ok;
     int32_t* err;
@@ -95,6 +104,15 @@ struct AttnArgs {
     // rotary embedding of q (null: q is used as given): table [rope_max_pos][D/2] float2 (cos, sin)
     const float2* rope;
     int32_t rope_max_pos;
+    // decode: partial-result rows per slot (16: one row per query head of a KV head)
+    int32_t rows_per_slot;
+    // decode over a shared prefix: the private items' page-table columns start at page0; the shared-prefix
+    // items (kGroup) each cover `group_agents` consecutive agents of one KV head over a piece of the
+    // shared_tiles shared KV tiles, their queries loaded through tm_qg (box {64, G, group_agents})
+    int32_t page0;
+    const int32_t* unit_slot;  // first partial slot of unit (agent b, KV head g) at b * Hkv + g
+    int32_t group_items, group_ns, group_agents, groups_per_head, shared_tiles, batch;
+    CUtensorMap tm_qg;
 };
 
 struct CombineArgs {
@@ -106,6 +124,7 @@ struct CombineArgs {
     const int32_t* cu;
     void* out;
     int32_t Hq, G, D, tq;
+    int32_t rows;          // partial rows per slot: kNQ * kBM (extend) or 16 (decode)
 };
 
 // Launch `kernel` so that it may start while the kernel before it on the stream finishes (programmatic
@@ -141,5 +160,8 @@ size_t extend_attention_smem_bytes(int head_dim);
 // Decode: the same arguments (tm_q boxes one token of G heads); units from the schedule run on
 // prefix = kv_lens - 1 and suffix = 1, which the schedule writes (SchedArgs::kv_lens).
 cudaError_t launch_decode_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st);
+// The shared-prefix items of rr_decode_attention_shared (a.group_items of them, one KV head x group_agents
+// agents x a piece of the shared tiles each); partial results into the agents' first unit slots.
+cudaError_t launch_decode_shared_prefix(const AttnArgs& a, int head_dim, int grid, cudaStream_t st);
 
 }  // namespace rr

@@ -104,11 +104,20 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     const int chunk = (B + 1023) / 1024;
     const int b0 = min(B, tid * chunk), b1 = min(B, b0 + chunk);
     if (a.kv_lens) {  // decode: the lengths in prefix / suffix form (read back below by the same threads,
-                      // and by every thread after the next barrier)
+                      // and by every thread after the next barrier); over a shared prefix, the private keys
         for (int b = b0; b < b1; ++b) {
-            const int L = a.kv_lens[b];
-            a.prefix_out[b] = L - 1;
+            const int L = a.kv_lens[b] - a.lens_offset;
+            a.prefix_out[b] = L - 1;  // L < 1 fails the check below
             a.suffix_out[b] = 1;
+        }
+        if (a.shared_pages > 0) {  // every agent's shared-prefix pages are agent 0's
+            for (long long i = tid; i < (long long)B * a.shared_pages; i += 1024) {
+                const long long b = i / a.shared_pages, p = i % a.shared_pages;
+                if (a.page_table[b * a.max_pages + p] != a.page_table[p]) {
+                    atomicCAS(a.err, 0, RR_ERR_SHARED);
+                    s_bad = 1;
+                }
+            }
         }
     }
     const long long cap = (long long)a.max_pages * a.ps;
@@ -188,8 +197,11 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     // `cost` KV tiles becomes ceil(cost / target) items (at most 64), target = total / (W waves), at
     // least 8 tiles.  Then items <= total/target + units <= (W + 2) waves, which bounds the partial buffers.
     const long long W = a.split_waves > 0 ? a.split_waves : 2;
-    const bool split = a.split_grid > 0 && tot_u < 2ll * a.split_grid && tot_u <= 1024 && tot_u > 0;
-    const long long target = split ? max(8ll, (tot_cost + W * a.split_grid - 1) / (W * a.split_grid)) : 0;
+    // extra_slots > 0 (decode over a shared prefix): every unit writes partials, split or not
+    const bool split = tot_u > 0 && tot_u <= 1024 &&
+                       (a.extra_slots > 0 || (a.split_grid > 0 && tot_u < 2ll * a.split_grid));
+    const bool cut = split && a.split_grid > 0 && tot_u < 2ll * a.split_grid;  // pieces per unit > 1 allowed
+    const long long target = cut ? max(8ll, (tot_cost + W * a.split_grid - 1) / (W * a.split_grid)) : (1ll << 40);
     int my_b = 0, my_g = 0, my_u = 0, my_ns = 1;
     long long my_unit_cost = 0;
     int my_cost32 = 0;  // the same, in 32 bits (a unit reads fewer than 2^24 tiles: 2^31 keys)
@@ -207,9 +219,11 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
         my_cost32 = (int)my_unit_cost;
     }
     // partial-result slots and the rank of each split unit (exclusive scans over units)
+    const bool my_partial = split && tid < tot_u && (my_ns > 1 || a.extra_slots > 0);
+    const int my_slots = my_partial ? my_ns + a.extra_slots : 0;
     long long my_slot_base = 0, my_rank = 0, n_slots = 0, n_split_units = 0;
-    block_exclusive_scan2(my_ns > 1 ? my_ns : 0, my_ns > 1 ? 1 : 0, my_slot_base, my_rank, n_slots, n_split_units,
-                          s_ws, s_wu);
+    block_exclusive_scan2(my_slots, my_partial ? 1 : 0, my_slot_base, my_rank, n_slots, n_split_units, s_ws, s_wu);
+    if (my_partial && a.unit_slot) a.unit_slot[(long long)my_b * a.Hkv + my_g] = (int32_t)my_slot_base;
 
     // ---- 3. histogram of item costs
     for (int i = tid; i < kCostBuckets; i += 1024) s_hist[i] = 0;
@@ -272,12 +286,14 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
             const int c = piece_tiles(my_cost32, my_ns, sp);
             const int pos = atomicAdd(&s_hist[min(c, kCostBuckets - 1)], 1);
             a.units[pos] = make_int4(my_b, my_g | (sp << 8) | (my_ns << 16), my_u, (int)my_unit_cost);
-            a.item_slot[pos] = my_ns > 1 ? (int)(my_slot_base + sp) : -1;
+            a.item_slot[pos] = my_partial ? (int)(my_slot_base + a.extra_slots + sp) : -1;
         }
-        if (my_ns > 1) a.split_units[my_rank] = make_int4(my_b, my_g | (my_ns << 16), my_u, (int)my_slot_base);
+        if (my_partial) a.split_units[my_rank] = make_int4(my_b, my_g | (my_slots << 16), my_u, (int)my_slot_base);
     }
     if (tid == 0) {
-        *a.n_units = split ? (int32_t)(n_slots + (tot_u - n_split_units)) : (int32_t)tot_u;
+        // items: the pieces of every unit (slots minus the reserved ones of units that write partials)
+        *a.n_units = split ? (int32_t)(n_slots - (long long)a.extra_slots * n_split_units + (tot_u - n_split_units))
+                           : (int32_t)tot_u;
         *a.n_split = split ? (int32_t)n_split_units : 0;
     }
 }
