@@ -10,9 +10,12 @@
 //   3. if the batch has fewer than two waves of units, split each unit's KV
 //      range into items (split-K) so the grid stays full; the partial results
 //      are merged by the combine kernel;
-//   4. counting-sort the items by cost, most expensive first, so a persistent
-//      grid that takes them in order approximates longest-processing-time
-//      scheduling.  This is what balances a batch whose agents have very
+//   4. order the items most expensive first, so a persistent grid that takes
+//      them in order approximates longest-processing-time scheduling: whole
+//      (agent, KV head) groups by their total cost with each group's units
+//      together (unsplit batches of up to 1024 groups; the units of a group
+//      then share their K/V pages through L2), else a counting sort of the
+//      items by cost.  This is what balances a batch whose agents have very
 //      different cached prefixes and uncached suffixes (the skew an eviction
 //      policy creates, Sec. 3.1-3.3).
 // Within a cost bucket the order is not fixed (atomics), which is harmless: a
@@ -92,6 +95,7 @@ __device__ void block_exclusive_scan2(long long x, long long y, long long& ex, l
 __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     __shared__ long long s_ws[32], s_wu[32];
     __shared__ int s_hist[kCostBuckets];
+    __shared__ long long s_key[1024];
     __shared__ int s_bad;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     // the consumer kernel may start its prologue now; it waits for this kernel before reading its output
@@ -224,6 +228,64 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     long long my_slot_base = 0, my_rank = 0, n_slots = 0, n_split_units = 0;
     block_exclusive_scan2(my_slots, my_partial ? 1 : 0, my_slot_base, my_rank, n_slots, n_split_units, s_ws, s_wu);
     if (my_partial && a.unit_slot) a.unit_slot[(long long)my_b * a.Hkv + my_g] = (int32_t)my_slot_base;
+
+    // ---- 3'. unsplit batches of at most 1024 (agent, KV head) groups: order the GROUPS by their total cost,
+    // most expensive first, and list each group's units together, most expensive first.  A wave's CTAs then
+    // work on the units of a few groups at once, which stream the same K/V pages at about the same time and
+    // share them through L2, instead of a group's units landing in different waves and reading its pages
+    // from DRAM again; the order stays longest-first at the granularity of groups, and is deterministic.
+    const long long n_groups = (long long)B * a.Hkv;
+    if (!split && n_groups <= 1024) {
+        long long gcost = 0;
+        if (tid < n_groups) {
+            const int b = tid / a.Hkv;
+            const int S = suffix[b], P = prefix[b];
+            const int nu = (S + a.unit_tokens - 1) / a.unit_tokens;
+            for (int u = 0; u < nu; ++u)
+                gcost += ((long long)P + min((long long)S, (long long)(u + 1) * a.unit_tokens) + kBN - 1) / kBN;
+        }
+        // key: cost, then the lower group index first on ties; empty slots sort below every group
+        s_key[tid] = tid < n_groups ? ((gcost << 10) | (1023 - tid)) : -1;
+        __syncthreads();
+        for (int k = 2; k <= 1024; k <<= 1) {  // bitonic sort, ascending
+            for (int j = k >> 1; j > 0; j >>= 1) {
+                const int ixj = tid ^ j;
+                if (ixj > tid) {
+                    const long long x = s_key[tid], y = s_key[ixj];
+                    if (((tid & k) == 0) ? (x > y) : (x < y)) {
+                        s_key[tid] = y;
+                        s_key[ixj] = x;
+                    }
+                }
+                __syncthreads();
+            }
+        }
+        // thread r takes the r-th most expensive group and writes its units from position start on
+        const long long key = s_key[1023 - tid];
+        int b = 0, h = 0, nu = 0;
+        if (key >= 0) {
+            const int gidx = 1023 - (int)(key & 1023);
+            b = gidx / a.Hkv;
+            h = gidx % a.Hkv;
+            nu = (suffix[b] + a.unit_tokens - 1) / a.unit_tokens;
+        }
+        long long start = 0, dummy = 0, t0 = 0, t1 = 0;
+        block_exclusive_scan2(nu, 0, start, dummy, t0, t1, s_ws, s_wu);
+        if (nu > 0) {
+            const int S = suffix[b], P = prefix[b];
+            for (int i = 0; i < nu; ++i) {
+                const int u = nu - 1 - i;
+                const long long n_keys = (long long)P + min((long long)S, (long long)(u + 1) * a.unit_tokens);
+                a.units[start + i] = make_int4(b, h | (1 << 16), u, (int)((n_keys + kBN - 1) / kBN));
+                a.item_slot[start + i] = -1;
+            }
+        }
+        if (tid == 0) {
+            *a.n_units = (int32_t)tot_u;
+            *a.n_split = 0;
+        }
+        return;
+    }
 
     // ---- 3. histogram of item costs
     for (int i = tid; i < kCostBuckets; i += 1024) s_hist[i] = 0;
