@@ -11,11 +11,11 @@
 //      range into items (split-K) so the grid stays full; the partial results
 //      are merged by the combine kernel;
 //   4. order the items most expensive first, so a persistent grid that takes
-//      them in order approximates longest-processing-time scheduling: whole
-//      (agent, KV head) groups by their total cost with each group's units
-//      together (unsplit batches of up to 1024 groups; the units of a group
-//      then share their K/V pages through L2), else a counting sort of the
-//      items by cost.  This is what balances a batch whose agents have very
+//      them in order approximates longest-processing-time scheduling: runs of
+//      up to 128 consecutive units of one (agent, KV head) kept together and
+//      ordered by their most expensive unit (unsplit batches of up to 1024
+//      groups: a run's units share their K/V pages through L2), else a
+//      counting sort of the items by cost.  This is what balances a batch whose agents have very
 //      different cached prefixes and uncached suffixes (the skew an eviction
 //      policy creates, Sec. 3.1-3.3).
 // Within a cost bucket the order is not fixed (atomics), which is harmless: a
@@ -95,7 +95,7 @@ __device__ void block_exclusive_scan2(long long x, long long y, long long& ex, l
 __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     __shared__ long long s_ws[32], s_wu[32];
     __shared__ int s_hist[kCostBuckets];
-    __shared__ long long s_key[1024];
+    __shared__ long long s_key[2048];
     __shared__ int s_bad;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     // the consumer kernel may start its prologue now; it waits for this kernel before reading its output
@@ -229,62 +229,89 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     block_exclusive_scan2(my_slots, my_partial ? 1 : 0, my_slot_base, my_rank, n_slots, n_split_units, s_ws, s_wu);
     if (my_partial && a.unit_slot) a.unit_slot[(long long)my_b * a.Hkv + my_g] = (int32_t)my_slot_base;
 
-    // ---- 3'. unsplit batches of at most 1024 (agent, KV head) groups: order the GROUPS by their total cost,
-    // most expensive first, and list each group's units together, most expensive first.  A wave's CTAs then
-    // work on the units of a few groups at once, which stream the same K/V pages at about the same time and
-    // share them through L2, instead of a group's units landing in different waves and reading its pages
-    // from DRAM again; the order stays longest-first at the granularity of groups, and is deterministic.
+    // ---- 3'. unsplit batches of at most 1024 (agent, KV head) groups: list the units of a group in runs of
+    // up to 128 consecutive units (a chunk), most expensive unit first, and order the chunks by their most
+    // expensive unit.  A wave's CTAs then work on a few chunks at once, whose units stream the same K/V pages
+    // at about the same time and share them through L2, instead of a group's units landing in different
+    // waves and reading its pages from DRAM again; and since chunks are ordered by unit cost, the list stays
+    // close to longest-first, which keeps the persistent grid's CTAs evenly loaded.  Deterministic.
     const long long n_groups = (long long)B * a.Hkv;
     if (!split && n_groups <= 1024) {
-        long long gcost = 0;
+        int nu = 0, P = 0, S = 0;  // group tid = (agent tid / Hkv, KV head tid % Hkv)
         if (tid < n_groups) {
-            const int b = tid / a.Hkv;
-            const int S = suffix[b], P = prefix[b];
-            const int nu = (S + a.unit_tokens - 1) / a.unit_tokens;
-            for (int u = 0; u < nu; ++u)
-                gcost += ((long long)P + min((long long)S, (long long)(u + 1) * a.unit_tokens) + kBN - 1) / kBN;
+            S = suffix[tid / a.Hkv];
+            P = prefix[tid / a.Hkv];
+            nu = (S + a.unit_tokens - 1) / a.unit_tokens;
         }
-        // key: cost, then the lower group index first on ties; empty slots sort below every group
-        s_key[tid] = tid < n_groups ? ((gcost << 10) | (1023 - tid)) : -1;
-        __syncthreads();
-        for (int k = 2; k <= 1024; k <<= 1) {  // bitonic sort, ascending
-            for (int j = k >> 1; j > 0; j >>= 1) {
-                const int ixj = tid ^ j;
-                if (ixj > tid) {
-                    const long long x = s_key[tid], y = s_key[ixj];
-                    if (((tid & k) == 0) ? (x > y) : (x < y)) {
-                        s_key[tid] = y;
-                        s_key[ixj] = x;
+        // the shortest chunk (128, 256 or 512 units) that keeps the batch within the sort's 2048 slots: a
+        // group longer than that (a long suffix, whose units' costs spread widely) is cut for balance, the
+        // others stay whole so that their units run in one wave
+        int run = 0;
+        for (int r = 128; r <= 512 && !run; r <<= 1)
+            if (block_sum((nu + r - 1) / r, s_ws) <= 2048) run = r;
+        if (run) {
+            const int nch = (nu + run - 1) / run;
+            long long cbase = 0, dummy = 0, t0 = 0, t1 = 0;
+            block_exclusive_scan2(nch, 0, cbase, dummy, t0, t1, s_ws, s_wu);
+            for (int i2 = tid; i2 < 2048; i2 += 1024) s_key[i2] = -1;  // empty slots sort below every chunk
+            __syncthreads();
+            for (int c = 0; c < nch; ++c) {  // chunk c: units nu-1-c*run down to max(0, nu-(c+1)*run)
+                const int u = nu - 1 - c * run;
+                const long long top = ((long long)P + min((long long)S, (long long)(u + 1) * a.unit_tokens) + kBN - 1) / kBN;
+                const long long id = ((long long)tid << 11) | c;  // group, chunk within it (< 2048)
+                s_key[cbase + c] = (top << 21) | ((1ll << 21) - 1 - id);  // by cost, then group and chunk order
+            }
+            __syncthreads();
+            for (int k = 2; k <= 2048; k <<= 1) {  // bitonic sort of 2048 keys, ascending, two per thread
+                for (int jj = k >> 1; jj > 0; jj >>= 1) {
+                    for (int i2 = tid; i2 < 2048; i2 += 1024) {
+                        const int ixj = i2 ^ jj;
+                        if (ixj > i2) {
+                            const long long x = s_key[i2], y = s_key[ixj];
+                            if (((i2 & k) == 0) ? (x > y) : (x < y)) {
+                                s_key[i2] = y;
+                                s_key[ixj] = x;
+                            }
+                        }
+                    }
+                    __syncthreads();
+                }
+            }
+            // thread t takes ranks 2t and 2t + 1 (rank 0 = the chunk with the most expensive unit)
+            int cg[2], cc[2], cn[2];
+            for (int q = 0; q < 2; ++q) {
+                const long long key = s_key[2047 - (2 * tid + q)];
+                cg[q] = -1; cc[q] = 0; cn[q] = 0;
+                if (key >= 0) {
+                    const long long id = (1ll << 21) - 1 - (key & ((1ll << 21) - 1));
+                    cg[q] = (int)(id >> 11);
+                    cc[q] = (int)(id & 2047);
+                    const int gnu = (suffix[cg[q] / a.Hkv] + a.unit_tokens - 1) / a.unit_tokens;
+                    cn[q] = min(run, gnu - cc[q] * run);
+                }
+            }
+            long long start = 0, d2 = 0, t2 = 0, t3 = 0;
+            block_exclusive_scan2(cn[0] + cn[1], 0, start, d2, t2, t3, s_ws, s_wu);
+            for (int q = 0; q < 2; ++q) {
+                if (cg[q] >= 0) {
+                    const int gb = cg[q] / a.Hkv, gh = cg[q] % a.Hkv;
+                    const int gS = suffix[gb], gP = prefix[gb];
+                    const int gnu = (gS + a.unit_tokens - 1) / a.unit_tokens;
+                    for (int i2 = 0; i2 < cn[q]; ++i2) {
+                        const int u = gnu - 1 - cc[q] * run - i2;
+                        const long long n_keys = (long long)gP + min((long long)gS, (long long)(u + 1) * a.unit_tokens);
+                        a.units[start + i2] = make_int4(gb, gh | (1 << 16), u, (int)((n_keys + kBN - 1) / kBN));
+                        a.item_slot[start + i2] = -1;
                     }
                 }
-                __syncthreads();
+                start += cn[q];
             }
-        }
-        // thread r takes the r-th most expensive group and writes its units from position start on
-        const long long key = s_key[1023 - tid];
-        int b = 0, h = 0, nu = 0;
-        if (key >= 0) {
-            const int gidx = 1023 - (int)(key & 1023);
-            b = gidx / a.Hkv;
-            h = gidx % a.Hkv;
-            nu = (suffix[b] + a.unit_tokens - 1) / a.unit_tokens;
-        }
-        long long start = 0, dummy = 0, t0 = 0, t1 = 0;
-        block_exclusive_scan2(nu, 0, start, dummy, t0, t1, s_ws, s_wu);
-        if (nu > 0) {
-            const int S = suffix[b], P = prefix[b];
-            for (int i = 0; i < nu; ++i) {
-                const int u = nu - 1 - i;
-                const long long n_keys = (long long)P + min((long long)S, (long long)(u + 1) * a.unit_tokens);
-                a.units[start + i] = make_int4(b, h | (1 << 16), u, (int)((n_keys + kBN - 1) / kBN));
-                a.item_slot[start + i] = -1;
+            if (tid == 0) {
+                *a.n_units = (int32_t)tot_u;
+                *a.n_split = 0;
             }
+            return;
         }
-        if (tid == 0) {
-            *a.n_units = (int32_t)tot_u;
-            *a.n_split = 0;
-        }
-        return;
     }
 
     // ---- 3. histogram of item costs
