@@ -236,7 +236,8 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     // waves and reading its pages from DRAM again; and since chunks are ordered by unit cost, the list stays
     // close to longest-first, which keeps the persistent grid's CTAs evenly loaded.  Deterministic.
     const long long n_groups = (long long)B * a.Hkv;
-    if (!split && n_groups <= 1024) {
+    // (decode: a group is one unit, so the counting sort below gives the same order, faster)
+    if (!split && n_groups <= 1024 && !a.kv_lens) {
         int nu = 0, P = 0, S = 0;  // group tid = (agent tid / Hkv, KV head tid % Hkv)
         if (tid < n_groups) {
             S = suffix[tid / a.Hkv];
