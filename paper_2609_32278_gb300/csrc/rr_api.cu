@@ -385,13 +385,13 @@ int decode_shared_impl(const void* q, const void* k_pool, const void* v_pool, co
     const int unit_tokens = rr::kNQ * tq;
     const int64_t units = B * Hkv;
     // shared-prefix items: one KV head x group_agents agents x one of group_ns pieces of the shared tiles;
-    // enough pieces for two waves
+    // enough pieces for two waves, but none shorter than 8 tiles (a piece's fixed cost would dominate)
     const int group_agents = 16 / G;
     const int64_t groups_per_head = (B + group_agents - 1) / group_agents;
     const int shared_tiles = shared_len / rr::kBN;
     const int64_t groups = groups_per_head * Hkv;
     const int group_ns = (int)std::max<int64_t>(
-        1, std::min<int64_t>(std::min(64, shared_tiles), (2ll * grid_sm + groups - 1) / groups));
+        1, std::min<int64_t>(std::min(64, std::max(1, shared_tiles / 8)), (2ll * grid_sm + groups - 1) / groups));
     const int split_waves = 6;
     // slots: every unit's group_ns shared pieces plus its private pieces (1 each, or a split into at most
     // (waves + 2) x grid pieces over all units)

@@ -191,3 +191,16 @@ def test_gpu_generator_matches_cpu(rr):
     t = synth.cpu_tensors(wl)
     for k in ("q", "k_new", "v_new", "k_pool", "v_pool"):
         np.testing.assert_array_equal(bf16_bits(g[k]), t[k])
+
+
+def test_more_groups_than_the_run_sort_takes(rr):
+    """More than 1024 (agent, KV head) groups: the schedule lists the units by a counting sort on their cost
+    instead of in per-group runs; every row against the oracle."""
+    rng = np.random.default_rng(31)
+    B = 300
+    P = rng.integers(0, 300, B)
+    S = rng.integers(1, 40, B)
+    wl = synth.custom("many_groups", B, 8, 4, 64, P, S, seed=31)
+    assert wl.B * wl.Hkv > 1024
+    out, _ = run_gpu(rr, wl)
+    check_close(to_f64(out), run_oracle(wl, 1.0 / math.sqrt(64)), "many_groups")
