@@ -327,6 +327,22 @@ const char* rr_last_error(void);
 /* Library version string. */
 const char* rr_version(void);
 
+/*
+ * rr_set_wait_limit -- the budget, in GPU clock cycles, of the pipeline waits
+ * of the attention kernels launched from now on by this process: every wait of
+ * the decode kernel, and in the extend kernel the waits of its stage watcher
+ * (the one thread that every K/V tile passes; the other roles keep the default
+ * budget).  cycles <= 0 restores the default (2^33, about 4 s at 2 GHz).  A
+ * wait that runs out does not trap: the kernel records RR_ERR_TIMEOUT in the
+ * device error word, every role of every CTA leaves at its next unfinished
+ * wait, in-flight copies and tensor-core operations are drained, tensor memory
+ * is freed and the kernel returns, so the context stays usable.  A budget far
+ * below a tile's load time makes that path run (the tests do this); results of
+ * such a call are undefined.  One try of a wait suspends the thread for at
+ * most a quarter of the budget (0.2 ms by default).
+ */
+void rr_set_wait_limit(long long cycles);
+
 /* Free the per-device workspaces (synchronises each device that has one). */
 void rr_shutdown(void);
 

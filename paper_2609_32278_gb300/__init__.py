@@ -44,7 +44,7 @@ RR_ERR_SHARED = 8
 EXPORTS = ("rr_kv_append", "rr_extend_attention", "rr_extend_step", "rr_decode_attention", "rr_validate_page_table",
            "rr_get_device_error", "rr_last_error", "rr_version", "rr_shutdown", "rr_extend_attention_noalloc",
            "rr_rope_table", "rr_kv_append_rope", "rr_extend_attention_rope", "rr_extend_step_rope",
-           "rr_decode_attention_rope", "rr_decode_attention_shared")
+           "rr_decode_attention_rope", "rr_decode_attention_shared", "rr_set_wait_limit")
 
 
 class RRError(RuntimeError):
@@ -106,6 +106,8 @@ def lib():
         L.rr_last_error.argtypes = []
         L.rr_version.restype = ctypes.c_char_p
         L.rr_version.argtypes = []
+        L.rr_set_wait_limit.restype = None
+        L.rr_set_wait_limit.argtypes = [ctypes.c_longlong]
         L.rr_shutdown.restype = None
         L.rr_shutdown.argtypes = []
         _lib = L
@@ -323,6 +325,13 @@ def validate_page_table(page_table, prefix_lens, suffix_lens, num_pages: int, pa
     T = int(sl.sum()) if total_tokens is None else int(total_tokens)
     dims = make_dims(len(pl), 1, 1, 64, page_size, pt.shape[1] if pt.ndim == 2 else 0, num_pages, T)
     return int(lib().rr_validate_page_table(pt.ctypes.data, pl.ctypes.data, sl.ctypes.data, ctypes.byref(dims)))
+
+
+def set_wait_limit(cycles: int) -> None:
+    """Budget in clock cycles of the decode kernel's pipeline waits and the extend kernel's stage-watcher
+    waits (<= 0: the default, ~4 s); a wait that runs out ends the kernel with RR_ERR_TIMEOUT in the
+    device error word (rr_set_wait_limit)."""
+    lib().rr_set_wait_limit(int(cycles))
 
 
 def last_error() -> str:

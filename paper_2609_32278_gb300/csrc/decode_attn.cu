@@ -60,7 +60,7 @@ constexpr int kDecWarpProducer = 4;
 constexpr int kDecWarpMMA = 5;
 constexpr int kHeadCols = 16;          // N of both MMAs: the G heads of a KV head, padded
 constexpr uint32_t kDecTmemCols = 64;  // S^T buffers at columns 0 and 16, O^T at 32
-constexpr long long kDecWaitLimit = 1ll << 33;  // ~4 s at 2 GHz
+constexpr long long kDecWaitLimit = 1ll << 33;  // ~4 s at 2 GHz: the TMEM release wait (pipeline waits: a.wait_limit)
 
 template <int D, int NS>
 struct DecCfg {
@@ -93,15 +93,17 @@ struct DecCfg {
 struct DecCtl {
     volatile int32_t* abort_flag;
     int32_t* err;
+    long long limit;  // cycles a pipeline wait may take before it gives up
+    uint32_t hint;    // ns a try may suspend the thread (less than the budget)
 };
 
 __device__ __forceinline__ bool dec_wait(uint32_t bar, uint32_t parity, const DecCtl& c) {
     if (ptx::mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
     for (;;) {
-        if (ptx::mbar_try_wait_sleep(bar, parity, 200000u)) return true;
+        if (ptx::mbar_try_wait_sleep(bar, parity, c.hint)) return true;
         if (*c.abort_flag) return false;
-        if (clock64() - t0 > kDecWaitLimit) {
+        if (clock64() - t0 > c.limit) {
             *c.abort_flag = 1;
             atomicCAS(c.err, 0, RR_ERR_TIMEOUT);
             return false;
@@ -225,7 +227,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
     const uint32_t sb = ptx::smem_u32(smem);
     auto bar = [&](int i) -> uint32_t { return sb + C::kOffBar + 8u * (uint32_t)i; };
     volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(smem + C::kOffMisc + 4);
-    const DecCtl ctl{abort_flag, a.err};
+    const DecCtl ctl{abort_flag, a.err, a.wait_limit, a.wait_hint_ns};
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     // Q^T rows G..15 and both P^T buffers start at zero: the padded head columns of S^T and O^T then

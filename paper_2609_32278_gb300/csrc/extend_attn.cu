@@ -113,15 +113,18 @@ struct Ctl {
 };
 
 // Bounded wait on an mbarrier phase.  False: timed out (flag raised) or another role aborted.
-// Each try may suspend the thread (up to 0.2 ms) until the phase completes, so waiting
-// warps leave the issue slots to the warps that are computing.
-__device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, const Ctl& c) {
+// Each try may suspend the thread (up to `hint` ns, 0.2 ms by default) until the phase completes,
+// so waiting warps leave the issue slots to the warps that are computing.  The stage watcher passes
+// the launch's budget (rr_set_wait_limit); the other roles keep the fixed one, which leaves their
+// code as it is, and leave at their next unfinished wait once any wait has run out.
+__device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, const Ctl& c,
+                                         long long limit = kWaitLimitCycles, uint32_t hint = 200000u) {
     if (ptx::mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
     for (;;) {
-        if (ptx::mbar_try_wait_sleep(bar, parity, 200000u)) return true;
+        if (ptx::mbar_try_wait_sleep(bar, parity, hint)) return true;
         if (*c.abort_flag) return false;
-        if (clock64() - t0 > kWaitLimitCycles) {
+        if (clock64() - t0 > limit) {
             *c.abort_flag = 1;
             atomicCAS(c.err, 0, RR_ERR_TIMEOUT);
             return false;
@@ -441,6 +444,8 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
         // ------------------------------------------------------------ stage watcher
         if (lane == 0) {
             uint32_t kv_count = 0, p_phase = 0;
+            const long long lim = a.wait_limit;
+            const uint32_t hint = a.wait_hint_ns;
             bool ok = true;
             for (int w = 0; ok; ++w) {
                 const int ui = unit_of(w, cta, grid);
@@ -450,12 +455,14 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                 const int n_kv = (sp + 1) * U.w / ns - sp * U.w / ns;
                 for (int j = 0; j < n_kv; ++j, ++kv_count) {
                     const uint32_t nxt = kv_count + 1;
-                    if (!(ok = wait_bar(bar(C::kVFull + (int)(kv_count % NV)), (kv_count / NV) & 1, ctl))) break;
-                    if (j + 1 < n_kv && !(ok = wait_bar(bar(C::kKFull + (int)(nxt % NK)), (nxt / NK) & 1, ctl)))
+                    if (!(ok = wait_bar(bar(C::kVFull + (int)(kv_count % NV)), (kv_count / NV) & 1, ctl, lim, hint)))
+                        break;
+                    if (j + 1 < n_kv &&
+                        !(ok = wait_bar(bar(C::kKFull + (int)(nxt % NK)), (nxt / NK) & 1, ctl, lim, hint)))
                         break;
                     ptx::mbar_arrive(bar(C::kPFull + 0));
                     // one arrival per phase: the next one only once this phase has completed
-                    if (!(ok = wait_bar(bar(C::kPFull + 0), p_phase, ctl))) break;
+                    if (!(ok = wait_bar(bar(C::kPFull + 0), p_phase, ctl, lim, hint))) break;
                     p_phase ^= 1u;
                 }
             }

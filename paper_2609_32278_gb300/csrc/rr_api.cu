@@ -4,6 +4,7 @@
 #include <cstdio>
 #include <algorithm>
 #include <cstring>
+#include <atomic>
 #include <mutex>
 #include <vector>
 
@@ -14,6 +15,7 @@
 namespace {
 
 thread_local char g_msg[512] = "";
+std::atomic<long long> g_wait_limit{0};  // 0: the default budget
 
 int fail(int code, const char* fmt, ...) {
     va_list ap;
@@ -175,6 +177,13 @@ int encode_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64
 
 }  // namespace
 
+namespace rr {
+long long wait_limit_cycles() {
+    const long long v = g_wait_limit.load(std::memory_order_relaxed);
+    return v > 0 ? v : (1ll << 33);
+}
+}  // namespace rr
+
 namespace {
 
 // Extend attention; decode attention (decode = true: kv_lens in place of the prefix / suffix lengths,
@@ -308,6 +317,8 @@ int attention_impl(const void* q, const void* k_pool, const void* v_pool, const 
     a.oob_row = (int32_t)rows;
     const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)D);
     a.scale_log2 = scale * 1.4426950408889634f;
+    a.wait_limit = rr::wait_limit_cycles();
+    a.wait_hint_ns = (uint32_t)std::min<long long>(200000, std::max<long long>(1, a.wait_limit / 4));
     const int64_t grid = std::min<int64_t>((int64_t)d->sm_count, max_items);
     if (fused) {
         // k_new / v_new [T][Hkv][D]: one row of Hkv * D per suffix token, the pool maps' box
@@ -469,6 +480,8 @@ int decode_shared_impl(const void* q, const void* k_pool, const void* v_pool, co
     a.oob_row = (int32_t)rows;
     const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)D);
     a.scale_log2 = scale * 1.4426950408889634f;
+    a.wait_limit = rr::wait_limit_cycles();
+    a.wait_hint_ns = (uint32_t)std::min<long long>(200000, std::max<long long>(1, a.wait_limit / 4));
     a.unit_slot = unit_slot;
     a.batch = (int32_t)B;
     // 1. the shared prefix, once per group of agents
@@ -509,6 +522,8 @@ extern "C" {
 const char* rr_version(void) { return "rr-extend 0.1 (sm_103a)"; }
 
 const char* rr_last_error(void) { return g_msg; }
+
+void rr_set_wait_limit(long long cycles) { g_wait_limit.store(cycles > 0 ? cycles : 0, std::memory_order_relaxed); }
 
 }  // extern "C"
 
@@ -903,6 +918,8 @@ extern "C" int rr_extend_attention_noalloc(const void* q, const void* k_pool, co
     a.oob_row = (int32_t)rows;
     const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)D);
     a.scale_log2 = scale * 1.4426950408889634f;
+    a.wait_limit = rr::wait_limit_cycles();
+    a.wait_hint_ns = (uint32_t)std::min<long long>(200000, std::max<long long>(1, a.wait_limit / 4));
     const int64_t grid = std::min<int64_t>((int64_t)sm_count, max_units);
     e = rr::launch_extend_attention(a, D, (int)std::max<int64_t>(grid, 1), stream);
     if (e != cudaSuccess) return cuda_fail(e, "extend attention kernel launch");

@@ -93,6 +93,9 @@ struct AttnArgs {
     int32_t tq;            // tokens per Q tile = 128 / G
     int32_t oob_row;       // first row past the pool (TMA fills it with zeros)
     float scale_log2;      // softmax scale * log2(e)
+    long long wait_limit;  // cycles a pipeline wait may take before the kernel gives up (RR_ERR_TIMEOUT):
+                           // every wait of the decode kernel, the extend kernel's stage watcher
+    uint32_t wait_hint_ns; // how long one try of such a wait may suspend the thread
     // fused extend step only (the suffix K/V is read from k_new / v_new and written to the pool here)
     CUtensorMap tm_knew;   // k_new [T][Hkv*D], box {64, ps}, 128B swizzle
     CUtensorMap tm_vnew;   // v_new, same
@@ -146,6 +149,9 @@ cudaError_t launch_after_sched(void (*kernel)(KArgs...), dim3 grid, dim3 block, 
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
 }
+
+// The pipeline wait budget the attention kernels get (rr_set_wait_limit; 2^33 cycles, ~4 s at 2 GHz, by default).
+long long wait_limit_cycles();
 
 cudaError_t launch_sched(const SchedArgs& a, cudaStream_t st);
 cudaError_t launch_combine(const CombineArgs& a, int grid, cudaStream_t st);
