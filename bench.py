@@ -641,7 +641,7 @@ def run_ours(args, world, rank, local):
     src_hash = kernel_source_hash()
     traffic_rec, _ = load_traffic(src_hash)
     traffic = None
-    if traffic_rec is not None and traffic_rec.get("workload") == args.config:
+    if traffic_rec is not None and traffic_rec.get("workload") == wl.name:  # the whole batch it was captured on, not a slice
         traffic = traffic_rec.get("dram_bytes_per_launch")
     roof = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16"], "unit": "TFLOP/s",
             "frac": achieved / peaks["bf16"], "traffic": traffic,
