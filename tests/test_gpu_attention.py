@@ -204,3 +204,29 @@ def test_more_groups_than_the_run_sort_takes(rr):
     assert wl.B * wl.Hkv > 1024
     out, _ = run_gpu(rr, wl)
     check_close(to_f64(out), run_oracle(wl, 1.0 / math.sqrt(64)), "many_groups")
+
+
+def test_batch_without_suffix_rows(rr):
+    """Every agent has S = 0 (T = 0): the extend call, the fused step (plain and rotary) and a decode over a
+    shared prefix with zero agents return empty outputs and OK, launch nothing that writes, and leave the
+    pool as it was."""
+    import torch
+    wl = synth.custom("no_rows", 3, 8, 2, 128, [32, 0, 300], [0, 0, 0], seed=33)
+    g = synth.gpu_tensors(wl, "cuda")
+    assert g["q"].shape[0] == 0
+    kp0, vp0 = bf16_bits(g["k_pool"]).copy(), bf16_bits(g["v_pool"]).copy()
+    out = rr.extend_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"], g["suffix_lens"])
+    assert out.shape == g["q"].shape
+    out = rr.extend_step(g["q"], g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                         g["suffix_lens"])
+    assert out.shape == g["q"].shape
+    table = rr.rope_table(400, wl.D, 500000.0, device=g["q"].device)
+    out = rr.extend_step(g["q"], g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                         g["suffix_lens"], rope=table)
+    assert out.shape == g["q"].shape
+    assert rr.device_error() == 0, rr.last_error()
+    assert np.array_equal(bf16_bits(g["k_pool"]), kp0) and np.array_equal(bf16_bits(g["v_pool"]), vp0)
+    empty = torch.zeros(0, dtype=torch.int32, device=g["q"].device)
+    out = rr.decode_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"][:0], empty, shared_len=128)
+    assert out.shape == g["q"].shape
+    assert rr.device_error() == 0, rr.last_error()
