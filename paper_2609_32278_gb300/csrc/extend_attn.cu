@@ -29,6 +29,8 @@
 //     P_1(j) is tested with a non-blocking mbarrier.test_wait issued in the
 //     same asm block as the last two MMAs of S_0(j+1), so the test's latency
 //     hides behind them; the blocking wait runs only if the phase was open.
+//     A unit's Q buffers are released with its last S GEMM, so the next unit's
+//     Q tiles load while the last PVs and softmax passes run.
 //   * warp 10, stage watcher (one thread): waits until V(j) and K(j+1) have
 //     landed and adds one arrival to P_0(j), so the MMA issuer's wait for
 //     P_0(j) covers both.  A wait on an mbarrier, even one already complete,
@@ -540,6 +542,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                     issue_qk(1, sk);
                     ptx::mma_commit(bar(C::kSFull + 1));
                     ptx::mma_commit(bar(C::kKEmpty + sk));
+                    if (n_kv == 1) ptx::mma_commit(bar(C::kQEmpty));  // Q is read by the S GEMMs only
                 }
                 // P_q waits: a test for the next P rides on the last MMAs of the S GEMM before it; the
                 // blocking wait runs only when that test found the phase still open.
@@ -566,12 +569,15 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                         const int qn = (q + 1) % kNQ;
                         p_ready[qn] = issue_qk_test(q, sk1, bar(C::kPFull + qn), (p_phase >> qn) & 1u);
                         ptx::mma_commit(bar(C::kSFull + q));
-                        if (q == kNQ - 1) ptx::mma_commit(bar(C::kKEmpty + sk1));
+                        if (q == kNQ - 1) {
+                            ptx::mma_commit(bar(C::kKEmpty + sk1));
+                            // the unit's last S GEMM: the next unit's Q may land while the last PVs run
+                            if (j + 2 == n_kv) ptx::mma_commit(bar(C::kQEmpty));
+                        }
                     }
                     if (!ok) break;
                 }
                 if (!ok) break;
-                ptx::mma_commit(bar(C::kQEmpty));
                 kv_count += n_kv;
                 ++unit_i;
             }
