@@ -95,8 +95,9 @@ __device__ void block_exclusive_scan2(long long x, long long y, long long& ex, l
 __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     __shared__ long long s_ws[32], s_wu[32];
     __shared__ int s_hist[kCostBuckets];
-    __shared__ long long s_key[2048];
+    __shared__ long long s_key[2048];  // run order: chunk keys; before that, the agents' unit offsets
     __shared__ int s_bad;
+    int32_t* s_uoff = reinterpret_cast<int32_t*>(s_key);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     // the consumer kernel may start its prologue now; it waits for this kernel before reading its output
     ptx::griddep_launch_dependents();
@@ -159,15 +160,22 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     long long off_s = (warp ? s_ws[warp - 1] : 0) + inc_s - sum_s;
     long long off_u = (warp ? s_wu[warp - 1] : 0) + inc_u - sum_u;
     const bool ok = !s_bad && tot_s == a.T && tot_s < (1ll << 31) && (!a.build_units || tot_u <= a.max_units);
+    // the binary searches below read the unit offsets from shared memory when they fit (B + 1 <= 4096)
+    const bool uoff_smem = B < 2 * 2048;
     if (ok) {
         for (int b = b0; b < b1; ++b) {
             const int S = a.suffix[b];
             a.cu[b] = (int32_t)off_s;
             a.unit_off[b] = (int32_t)off_u;
+            if (uoff_smem) s_uoff[b] = (int32_t)off_u;
             off_s += S;
             off_u += (long long)a.Hkv * ((S + a.unit_tokens - 1) / a.unit_tokens);
         }
-        if (tid == 0) { a.cu[B] = (int32_t)tot_s; a.unit_off[B] = (int32_t)tot_u; }
+        if (tid == 0) {
+            a.cu[B] = (int32_t)tot_s;
+            a.unit_off[B] = (int32_t)tot_u;
+            if (uoff_smem) s_uoff[B] = (int32_t)tot_u;
+        }
     }
     if (!ok) {
         if (tid == 0) {
@@ -183,20 +191,9 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     __syncthreads();  // every thread's cu / unit_off entries are written
     const int32_t* prefix = a.prefix;
     const int32_t* suffix = a.suffix;
-    const int32_t* unit_off = a.unit_off;
+    const int32_t* unit_off = uoff_smem ? s_uoff : a.unit_off;
 
-    // ---- 2. unit costs and their total (the split decision needs it)
-    long long my_cost = 0;
-    for (long long idx = tid; idx < tot_u; idx += 1024) {
-        const int b = last_le(unit_off, B, idx);
-        const int S = suffix[b], P = prefix[b];
-        const int nu = (S + a.unit_tokens - 1) / a.unit_tokens;
-        const int u = (int)(idx - unit_off[b]) % nu;
-        const long long n_keys = (long long)P + min((long long)S, (long long)(u + 1) * a.unit_tokens);
-        my_cost += (n_keys + kBN - 1) / kBN;
-    }
-    const long long tot_cost = block_sum(my_cost, s_ws);
-
+    // ---- 2. split decision: a unit's cost is the number of 128-key tiles its last row reads.
     // Split the KV range of every unit when the batch has fewer than two waves of units: a unit of
     // `cost` KV tiles becomes ceil(cost / target) items (at most 64), target = total / (W waves), at
     // least 8 tiles.  Then items <= total/target + units <= (W + 2) waves, which bounds the partial buffers.
@@ -205,11 +202,10 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     const bool split = tot_u > 0 && tot_u <= 1024 &&
                        (a.extra_slots > 0 || (a.split_grid > 0 && tot_u < 2ll * a.split_grid));
     const bool cut = split && a.split_grid > 0 && tot_u < 2ll * a.split_grid;  // pieces per unit > 1 allowed
-    const long long target = cut ? max(8ll, (tot_cost + W * a.split_grid - 1) / (W * a.split_grid)) : (1ll << 40);
     int my_b = 0, my_g = 0, my_u = 0, my_ns = 1;
     long long my_unit_cost = 0;
     int my_cost32 = 0;  // the same, in 32 bits (a unit reads fewer than 2^24 tiles: 2^31 keys)
-    if (split && tid < tot_u) {  // one unit per thread
+    if (split && tid < tot_u) {  // a split batch has at most 1024 units: one per thread
         my_b = last_le(unit_off, B, tid);
         const int S = suffix[my_b], P = prefix[my_b];
         const int nu = (S + a.unit_tokens - 1) / a.unit_tokens;
@@ -218,9 +214,13 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
         my_u = local % nu;
         const long long n_keys = (long long)P + min((long long)S, (long long)(my_u + 1) * a.unit_tokens);
         my_unit_cost = (n_keys + kBN - 1) / kBN;
+        my_cost32 = (int)my_unit_cost;
+    }
+    const long long tot_cost = cut ? block_sum(my_unit_cost, s_ws) : 0;  // `cut` is uniform over the block
+    const long long target = cut ? max(8ll, (tot_cost + W * a.split_grid - 1) / (W * a.split_grid)) : (1ll << 40);
+    if (split && tid < tot_u) {
         my_ns = (int)min(min(64ll, my_unit_cost), (my_unit_cost + target - 1) / target);
         if (my_ns < 1) my_ns = 1;
-        my_cost32 = (int)my_unit_cost;
     }
     // partial-result slots and the rank of each split unit (exclusive scans over units)
     const bool my_partial = split && tid < tot_u && (my_ns > 1 || a.extra_slots > 0);
@@ -254,7 +254,9 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
             const int nch = (nu + run - 1) / run;
             long long cbase = 0, dummy = 0, t0 = 0, t1 = 0;
             block_exclusive_scan2(nch, 0, cbase, dummy, t0, t1, s_ws, s_wu);
-            for (int i2 = tid; i2 < 2048; i2 += 1024) s_key[i2] = -1;  // empty slots sort below every chunk
+            int n2 = 2;  // sort length: the chunks rounded up to a power of two (<= 2048)
+            while (n2 < t0) n2 <<= 1;
+            for (int i2 = tid; i2 < n2; i2 += 1024) s_key[i2] = -1;  // empty slots sort below every chunk
             __syncthreads();
             for (int c = 0; c < nch; ++c) {  // chunk c: units nu-1-c*run down to max(0, nu-(c+1)*run)
                 const int u = nu - 1 - c * run;
@@ -263,9 +265,9 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
                 s_key[cbase + c] = (top << 21) | ((1ll << 21) - 1 - id);  // by cost, then group and chunk order
             }
             __syncthreads();
-            for (int k = 2; k <= 2048; k <<= 1) {  // bitonic sort of 2048 keys, ascending, two per thread
+            for (int k = 2; k <= n2; k <<= 1) {  // bitonic sort of n2 keys, ascending
                 for (int jj = k >> 1; jj > 0; jj >>= 1) {
-                    for (int i2 = tid; i2 < 2048; i2 += 1024) {
+                    for (int i2 = tid; i2 < n2; i2 += 1024) {
                         const int ixj = i2 ^ jj;
                         if (ixj > i2) {
                             const long long x = s_key[i2], y = s_key[ixj];
@@ -281,7 +283,8 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
             // thread t takes ranks 2t and 2t + 1 (rank 0 = the chunk with the most expensive unit)
             int cg[2], cc[2], cn[2];
             for (int q = 0; q < 2; ++q) {
-                const long long key = s_key[2047 - (2 * tid + q)];
+                const int rank = 2 * tid + q;
+                const long long key = rank < n2 ? s_key[n2 - 1 - rank] : -1;
                 cg[q] = -1; cc[q] = 0; cn[q] = 0;
                 if (key >= 0) {
                     const long long id = (1ll << 21) - 1 - (key & ((1ll << 21) - 1));
