@@ -57,11 +57,16 @@ def append_bytes(wl) -> float:
     return 4.0 * wl.T * wl.Hkv * wl.D * 2
 
 
-def kernel_source_hash() -> str:
-    """Hash of the attention kernel's code: comments, blank lines and indentation are left out, so an
-    edit to the comments keeps a recorded ncu figure valid and any code change invalidates it."""
+# the sources a kernel's DRAM traffic depends on: its own code and the schedule's unit order
+ATTN_SOURCES = ("extend_attn.cu", "ptx.cuh", "rope.cuh", "rr_internal.h", "sched.cu")
+DECODE_SOURCES = ("decode_attn.cu", "ptx.cuh", "rope.cuh", "rr_internal.h", "sched.cu")
+
+
+def kernel_source_hash(files=ATTN_SOURCES) -> str:
+    """Hash of a kernel's code: comments, blank lines and indentation are left out, so an edit to the
+    comments keeps a recorded ncu figure valid and any code change invalidates it."""
     h = hashlib.sha256()
-    for f in ("extend_attn.cu", "ptx.cuh", "rope.cuh", "rr_internal.h"):
+    for f in files:
         with open(os.path.join(ROOT, "paper_2609_32278_gb300", "csrc", f), encoding="utf-8") as fh:
             for line in fh:
                 code = line.split("//", 1)[0].strip()
@@ -229,9 +234,9 @@ def run_reference(args, world, rank):
     return 0
 
 
-def load_traffic(src_hash):
-    """DRAM bytes per attention launch from the committed ncu summary, if it was taken on this kernel source."""
-    path = os.path.join(ROOT, "profiles", "extend_attn_traffic.json")
+def load_traffic(src_hash, record="extend_attn_traffic.json"):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on this kernel source."""
+    path = os.path.join(ROOT, "profiles", record)
     try:
         with open(path) as f:
             rec = json.load(f)
@@ -315,13 +320,16 @@ def decode_leg(args, rr, synth, dev, st, peaks, rank):
     ms = statistics.mean(e0.elapsed_time(e1) for e0, e1 in ev)
     nbytes = decode_bytes(wl)
     gbs = nbytes / (ms * 1e-3) / 1e9
+    dec_hash = kernel_source_hash(DECODE_SOURCES)
+    rec, _ = load_traffic(dec_hash, "decode_attn_traffic.json")
+    traffic = rec.get("dram_bytes_per_launch") if rec is not None and rec.get("workload") == wl.name else None
     res = {"workload": wl.name, "B": wl.B, "Hq": wl.Hq, "Hkv": wl.Hkv, "D": wl.D,
            "kv_tokens": int((wl.prefix_lens.astype(np.int64) + 1).sum()), "calls": n, "ms_per_call": ms,
            "tokens_per_s": wl.B / (ms * 1e-3),
            "roofline": {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm"], "unit": "GB/s",
-                        "frac": gbs / peaks["hbm"], "traffic": None, "algorithmic_bytes": nbytes,
+                        "frac": gbs / peaks["hbm"], "traffic": traffic, "algorithmic_bytes": nbytes,
                         "kernel": f"decode_attn_kernel<{wl.D},{3 if wl.D == 128 else 6},{wl.G}>",
-                        "peak_kind": f"{peaks['src']} HBM copy bandwidth"},
+                        "peak_kind": f"{peaks['src']} HBM copy bandwidth", "kernel_source_hash": dec_hash},
            "l2": f"K/V working set {nbytes / 1e9:.1f} GB > 129 MB"}
     # a batch over a common prefix: the same calls through rr_decode_attention_shared (the shared pages read
     # once per group of 16 / G agents), checked against the plain call's output within the parity bar
