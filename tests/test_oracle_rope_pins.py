@@ -11,7 +11,7 @@ against something other than the oracle's own formula:
   rotation by p radians (complex multiplication by e^(ip)); a unit vector stays in its own pair and
   turns towards + the upper half; the frequency of pair i worked out by hand for D = 8, base 10^4;
   rotations compose (p then q equals p + q); scores depend on the relative position only;
-* rotated extend attention against a dense brute force that rotates through complex numbers and masks
+* rotated extend attention and rotated decode against a dense brute force that rotates through complex numbers and masks
   with an explicit matrix; a P = 0 agent's first key is stored unrotated, bit for bit.
 """
 import math
@@ -218,5 +218,20 @@ def test_rope_attention_single_key_is_value():
     kp, vp = oracle.kv_append_rope(t["k_new"], t["v_new"], t["k_pool"], t["v_pool"], wl.page_table,
                                    wl.prefix_lens, wl.suffix_lens, BASE)
     got = oracle.extend_attention_rope(t["q"], kp, vp, wl.page_table, wl.prefix_lens, wl.suffix_lens, BASE)
+    v = oracle.widen_bf16(t["v_new"])[0]
+    assert np.array_equal(got[0], np.repeat(v, 4, axis=0))
+
+
+def test_rope_decode_matches_dense_brute_force():
+    """Rotated decode (one new token per agent, its query rotated at L - 1) against the same dense brute
+    force: the last row of rotated causal attention over the agent's L keys."""
+    L = np.array([1, 40, 130])
+    wl = synth.custom("rope_dec", 3, 8, 2, 64, L - 1, np.ones(3, dtype=np.int64), seed=23)
+    t = synth.cpu_tensors(wl)
+    kp, vp = oracle.kv_append_rope(t["k_new"], t["v_new"], t["k_pool"], t["v_pool"], wl.page_table,
+                                   wl.prefix_lens, wl.suffix_lens, BASE)
+    got = oracle.decode_attention_rope(t["q"], kp, vp, wl.page_table, L.astype(np.int32), BASE)
+    np.testing.assert_allclose(got, _brute_force_rope(wl, BASE), atol=1e-11, rtol=0)
+    # the one-key agent (position 0: no rotation) returns its value exactly
     v = oracle.widen_bf16(t["v_new"])[0]
     assert np.array_equal(got[0], np.repeat(v, 4, axis=0))
