@@ -11,8 +11,9 @@ against something other than the oracle's own formula:
   rotation by p radians (complex multiplication by e^(ip)); a unit vector stays in its own pair and
   turns towards + the upper half; the frequency of pair i worked out by hand for D = 8, base 10^4;
   rotations compose (p then q equals p + q); scores depend on the relative position only;
-* rotated extend attention and rotated decode against a dense brute force that rotates through complex numbers and masks
-  with an explicit matrix; a P = 0 agent's first key is stored unrotated, bit for bit.
+* rotated extend attention and rotated decode against a dense brute force that rotates through
+  complex numbers and masks with an explicit matrix; a P = 0 agent's first key is stored unrotated,
+  bit for bit.
 """
 import math
 
