@@ -236,3 +236,30 @@ def test_rope_decode_matches_dense_brute_force():
     # the one-key agent (position 0: no rotation) returns its value exactly
     v = oracle.widen_bf16(t["v_new"])[0]
     assert np.array_equal(got[0], np.repeat(v, 4, axis=0))
+
+
+def test_round_bf16_special_values():
+    """Values the bf16 format fixes at the ends of its range: the largest finite value 0x7F7F =
+    (2 - 2^-7) 2^127; the tie halfway to 2^128 rounds to even, i.e. up to infinity (0x7F80), just below
+    it stays finite; signed zero, infinities and NaN (quiet, 0x7FC0) keep their kind."""
+    big = (2.0 - 2.0 ** -7) * 2.0 ** 127
+    cases = [
+        (big, 0x7F7F),
+        ((2.0 - 2.0 ** -8) * 2.0 ** 127, 0x7F80),                 # tie above the largest finite value
+        ((2.0 - 2.0 ** -8 - 2.0 ** -20) * 2.0 ** 127, 0x7F7F),    # just below the tie
+        (-big, 0xFF7F),
+        (-0.0, 0x8000),
+        (float("inf"), 0x7F80),
+        (float("-inf"), 0xFF80),
+        (2.0 ** -126, 0x0080),                                     # smallest normal
+        (2.0 ** -133, 0x0001),                                     # smallest subnormal
+    ]
+    got = oracle.round_bf16(np.array([c[0] for c in cases]))
+    assert [int(g) for g in got] == [c[1] for c in cases]
+    nan = int(oracle.round_bf16(np.array([float("nan")]))[0])
+    assert nan & 0x7F80 == 0x7F80 and nan & 0x007F != 0            # a NaN pattern
+
+
+def test_rope_rejects_odd_head_dim():
+    with pytest.raises(oracle.OracleError):
+        oracle.rope(np.zeros((2, 1, 7)), [0, 1], 10000.0)
