@@ -299,7 +299,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             const int t0 = u * unit_tokens;
             const int n_keys = P + min(S, t0 + unit_tokens);
             const int agent_len = P + S;
-            // Q tiles of this unit
+            // Q tiles of this unit, once the previous unit's last S GEMM has read its own (QEmpty)
             if (lane == 0) {
                 if (unit_i > 0) ok = wait_bar(bar(C::kQEmpty), (unit_i - 1) & 1, ctl);
                 if (ok) {
