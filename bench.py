@@ -222,7 +222,8 @@ def run_reference(args, world, rank):
         "impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": tm / args.steps * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": wl.name, "B": wl.B, "Hq": wl.Hq, "Hkv": wl.Hkv, "D": wl.D, "page_size": wl.ps,
+        "config": {"workload": wl.name, "inputs_sha256": wl.manifest()["sha256"][:16], "B": wl.B, "Hq": wl.Hq,
+                   "Hkv": wl.Hkv, "D": wl.D, "page_size": wl.ps,
                    "uncached_tokens": wl.T},
         "uncached_suffix_tokens_per_s": tok_per_s,
         "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": threads, "kind": "oracle",
@@ -323,7 +324,8 @@ def decode_leg(args, rr, synth, dev, st, peaks, rank):
     dec_hash = kernel_source_hash(DECODE_SOURCES)
     rec, _ = load_traffic(dec_hash, "decode_attn_traffic.json")
     traffic = rec.get("dram_bytes_per_launch") if rec is not None and rec.get("workload") == wl.name else None
-    res = {"workload": wl.name, "B": wl.B, "Hq": wl.Hq, "Hkv": wl.Hkv, "D": wl.D,
+    res = {"workload": wl.name, "inputs_sha256": wl.manifest()["sha256"][:16], "B": wl.B, "Hq": wl.Hq,
+           "Hkv": wl.Hkv, "D": wl.D,
            "kv_tokens": int((wl.prefix_lens.astype(np.int64) + 1).sum()), "calls": n, "ms_per_call": ms,
            "tokens_per_s": wl.B / (ms * 1e-3),
            "roofline": {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm"], "unit": "GB/s",
@@ -664,7 +666,8 @@ def run_ours(args, world, rank, local):
         "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": wl.name, "B": wl.B, "Hq": wl.Hq, "Hkv": wl.Hkv, "D": wl.D, "page_size": wl.ps,
+        "config": {"workload": wl.name, "inputs_sha256": wl.manifest()["sha256"][:16], "B": wl.B, "Hq": wl.Hq,
+                   "Hkv": wl.Hkv, "D": wl.D, "page_size": wl.ps,
                    "uncached_tokens": wl.T, "kv_tokens": int((wl.prefix_lens + wl.suffix_lens).sum()),
                    "num_pages": wl.num_pages, "l2": "inputs larger than L2 (KV working set "
                    f"{attn_bytes(wl) / 1e9:.1f} GB > 129 MB)", "parallelism": f"replicas x{world}"},

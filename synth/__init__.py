@@ -18,6 +18,8 @@ from __future__ import annotations
 
 import ctypes
 import dataclasses
+import hashlib
+import json
 import os
 import subprocess
 from typing import Dict, Optional
@@ -163,6 +165,29 @@ class Workload:
         cu = np.zeros(self.B + 1, dtype=np.int64)
         np.cumsum(self.suffix_lens.astype(np.int64), out=cu[1:])
         return cu
+
+    def manifest(self) -> Dict[str, object]:
+        """What makes this batch reproducible: its name, seed and shapes, the per-agent lengths and a
+        SHA-256 of the lengths and the page table (the tensor values are a pure function of the seed and
+        the logical coordinates, so these fix every input byte)."""
+        h = hashlib.sha256()
+        for a in (self.prefix_lens, self.suffix_lens, self.page_table):
+            arr = np.ascontiguousarray(a, dtype=np.int32)
+            h.update(str(arr.shape).encode())
+            h.update(arr.tobytes())
+        return {"name": self.name, "seed": int(self.seed), "B": int(self.B), "Hq": int(self.Hq),
+                "Hkv": int(self.Hkv), "D": int(self.D), "page_size": int(self.ps), "num_pages": int(self.num_pages),
+                "max_pages": self.max_pages, "shared_len": int(self.shared_len), "T": self.T,
+                "prefix_lens": [int(x) for x in self.prefix_lens], "suffix_lens": [int(x) for x in self.suffix_lens],
+                "sha256": h.hexdigest()}
+
+    def write_manifest(self, path: str) -> str:
+        """Write manifest() as JSON; returns its sha256."""
+        m = self.manifest()
+        with open(path, "w") as f:
+            json.dump(m, f, indent=1)
+            f.write("\n")
+        return str(m["sha256"])
 
     def row_agent_pos(self):
         """(agent, absolute position) of every suffix row, in q's row order."""

@@ -92,3 +92,19 @@ def test_config_shapes_follow_their_recipes():
     assert np.all(c5.page_table[:, :256] == c5.page_table[0, :256])
     c4 = synth.config("c4_coding")
     assert c4.G == 8 and np.all((c4.prefix_lens >= 131072) & (c4.prefix_lens <= 262144))
+
+
+def test_manifest_fixes_the_inputs(tmp_path):
+    """The manifest names everything the inputs depend on: the same config and seed give the same hash,
+    another seed (another page placement) or another config a different one; written to JSON it reads back."""
+    import json
+    a = synth.config("c2_llama3_8b", seed=0).manifest()
+    assert a == synth.config("c2_llama3_8b", seed=0).manifest()
+    assert a["sha256"] != synth.config("c2_llama3_8b", seed=1).manifest()["sha256"]
+    assert a["sha256"] != synth.config("c3_rr", seed=0).manifest()["sha256"]
+    assert a["T"] == sum(a["suffix_lens"]) and len(a["prefix_lens"]) == a["B"] == 32
+    wl = synth.custom("m", 2, 8, 2, 64, [16, 0], [5, 7], seed=3)
+    path = tmp_path / "m.json"
+    h = wl.write_manifest(str(path))
+    back = json.loads(path.read_text())
+    assert back["sha256"] == h and back["prefix_lens"] == [16, 0] and back["suffix_lens"] == [5, 7]
