@@ -545,7 +545,9 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
                 }
 #pragma unroll
                 for (int h = 0; h < G; ++h) {
-                    p[h] = ptx::ex2_approx(fmaf(x[h], sl2, -m[h]));  // x = -inf: p = 0
+                    // x = -inf: p = 0.  p is rounded to bf16 here, so the weight sum and the P^T operand of
+                    // the O^T GEMM hold the same weights and the output is a convex combination of V.
+                    p[h] = __bfloat162float(__float2bfloat16_rn(ptx::ex2_approx(fmaf(x[h], sl2, -m[h]))));
                     lp[h] += p[h];
                 }
                 // P^T(gt) goes to buffer buf once O^T(gt-2) has read it

@@ -176,6 +176,7 @@ __device__ __forceinline__ void exp2_poly2(float& p0, float& p1, float x0, float
 #endif
 constexpr int kEmuPairStride = RR_EMU_PAIR_STRIDE;
 
+
 // Snake order: even waves left to right, odd waves right to left.
 __device__ __forceinline__ int unit_of(int wave, int cta, int grid) {
     return wave * grid + ((wave & 1) ? (grid - 1 - cta) : cta);
@@ -728,9 +729,8 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                     m_run = mxs;
                 }
                 const float neg = m_run == -INFINITY ? 0.f : -m_run;  // a fully masked row keeps p = 0
-                // p = 2^(s * scale * log2e - m): packed FMA, ex2, packed accumulation over 8 chains; the
-                // first half of P goes to TMEM while the second is computed
-                float la[4] = {0.f, 0.f, 0.f, 0.f}, lb[4] = {0.f, 0.f, 0.f, 0.f};
+                // p = 2^(s * scale * log2e - m): packed FMA, ex2, bf16 pairs; the first half of P goes to TMEM
+                // while the second is computed
                 uint32_t pk[kBN / 2];
 #pragma unroll
                 for (int c = 0; c < kBN; c += 2) {
@@ -743,18 +743,10 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                         p0 = ptx::ex2_approx(x0);
                         p1 = ptx::ex2_approx(x1);
                     }
-                    const int k = (c >> 1) & 3;
-                    ptx::add2(la[k], lb[k], la[k], lb[k], p0, p1);
                     pk[c >> 1] = ptx::pack_bf16x2(p0, p1);
                     if (c == kBN / 2 - 2) ptx::tmem_st32(t_s, *reinterpret_cast<uint32_t(*)[32]>(&pk[0]));
                 }
                 ptx::tmem_st32(t_s + 32, *reinterpret_cast<uint32_t(*)[32]>(&pk[32]));
-                {
-                    float s0, s1, s2, s3;
-                    ptx::add2(s0, s1, la[0], lb[0], la[1], lb[1]);
-                    ptx::add2(s2, s3, la[2], lb[2], la[3], lb[3]);
-                    l_run += (s0 + s2) + (s1 + s3);
-                }
                 // O_q holds PV of tiles < j (complete: S_q(j) was issued after PV_q(j-1)); bring it to the
                 // new max before PV_q(j) may start, i.e. before this thread signals P_q(j).
                 if (__any_sync(0xffffffffu, grow)) {  // warp-uniform: tcgen05.ld/st are .sync.aligned
@@ -771,6 +763,23 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                 ptx::tmem_wait_st();
                 ptx::tc_fence_before();
                 ptx::mbar_arrive(bar(C::kPFull + q));
+                // The weight sum, from the same bf16 weights the PV product multiplies (each half of a packed
+                // pair widened exactly to f32), so that O / l is a convex combination of V rows.  It runs after
+                // P is signalled, off the softmax-to-MMA chain that bounds the kernel.  Against a sum of the
+                // unrounded f32 weights inside the chain this costs ~2 % of the attention time (c2 +1.9 %, c4
+                // +2.3 %); widening by mixed-precision adds instead cost +3.3 % / +4.0 %, and either inside the
+                // chain +5-10 %.
+                {
+                    float la[4] = {0.f, 0.f, 0.f, 0.f}, lb[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                    for (int c = 0; c < kBN / 2; ++c)
+                        ptx::add2(la[c & 3], lb[c & 3], la[c & 3], lb[c & 3], __uint_as_float(pk[c] << 16),
+                                  __uint_as_float(pk[c] & 0xFFFF0000u));
+                    float s0, s1, s2, s3;
+                    ptx::add2(s0, s1, la[0], lb[0], la[1], lb[1]);
+                    ptx::add2(s2, s3, la[2], lb[2], la[3], lb[3]);
+                    l_run += (s0 + s2) + (s1 + s3);
+                }
             }
             if (!ok) break;
             if (!(ok = wait_bar(bar(C::kOFinal + q), o_phase, ctl))) break;

@@ -168,3 +168,18 @@ def test_decode_rejects_bad_arguments(rr):
     # and the library still works afterwards
     out, _ = run_decode(rr, wl)
     assert np.isfinite(to_f64(out)).all()
+
+
+@pytest.mark.parametrize("L", [[2, 3, 4, 5], [130, 20000]], ids=["few_keys", "split"])
+def test_decode_unit_values_give_unit_output(rr, L):
+    """V == 1: the weight sum and the P^T operand hold the same bf16-rounded weights, so every output is 1 up
+    to fp32 summation order, which rounds to exactly 1.0 in bf16 (the second batch splits its key range and
+    goes through the combine)."""
+    wl = decode_workload("ones", len(L), 8, 2, 128, L)
+    g = synth.gpu_tensors(wl, "cuda")
+    g["v_new"].fill_(1.0)
+    for b in range(wl.B):
+        for lp in range(-(-int(wl.prefix_lens[b]) // wl.ps)):
+            g["v_pool"][int(wl.page_table[b, lp])] = 1.0
+    out, _ = run_decode(rr, wl, g=g)
+    np.testing.assert_array_equal(to_f64(out), 1.0)
