@@ -274,9 +274,9 @@ int rr_decode_attention_rope(const void* q, const void* k_pool, const void* v_po
  * device-wide synchronisation of cudaMalloc/cudaFree.  This entry point
  * computes exactly what rr_extend_attention computes (same kernels, same
  * arguments and layouts), but keeps its schedule scratch in one fixed array
- * of static device memory (about 1.31 MiB) that every GPU loading the library
- * holds until the process exits.  It calls no cudaMalloc, cudaFree or other
- * allocating routine.
+ * of static device memory (1,344,256 bytes, ~1.28 MiB) that every GPU
+ * loading the library holds until the process exits.  It calls no
+ * cudaMalloc, cudaFree or other allocating routine.
  *
  * Limits: at most 4096 agents, and at most 65536 schedule work units, where
  * the units needed are bounded by Hkv * (T / (256 / G) + B + 1).  Larger
@@ -345,6 +345,54 @@ void rr_set_wait_limit(long long cycles);
 
 /* Free the per-device workspaces (synchronises each device that has one). */
 void rr_shutdown(void);
+
+/*
+ * Self-describing tensors: the two calls of the extend step (rr_kv_append and
+ * rr_extend_attention, Sec. 2) with every argument carrying its shape,
+ * strides and element type, so that the library itself checks layouts a
+ * caller might get wrong (a strided view, a transposed pool, an int64 length
+ * array) instead of trusting the documented ones.  The plain-pointer calls
+ * above stay the primary form: their sizes travel in one rr_dims and their
+ * layouts are fixed by this header, which costs no per-call checks.
+ *
+ *   data    device pointer (same alignment rules as the plain calls)
+ *   ndim    number of dimensions (1 to 4)
+ *   shape   extent of each dimension, outermost first
+ *   stride  distance in ELEMENTS between consecutive indices of each
+ *           dimension; a dimension of extent 1 may have any stride
+ *   dtype   RR_DTYPE_BF16 or RR_DTYPE_I32
+ *
+ * Accepted layouts are the plain calls' ones, row-major and contiguous:
+ *   q, out [T, Hq, D] bf16; k_new, v_new [T, Hkv, D] bf16;
+ *   k_pool, v_pool [num_pages, ps, Hkv, D] bf16 (same shape);
+ *   page_table [B, max_pages] int32; prefix_lens, suffix_lens [B] int32.
+ * Errors, returned before anything is launched: a null tensor or data
+ * pointer, a wrong ndim, a negative extent or shapes that disagree with each
+ * other -> RR_ERR_INVALID_ARG; a wrong dtype or any stride other than
+ * row-major contiguous -> RR_ERR_UNSUPPORTED.  rr_last_error() names the
+ * argument and the dimension.  Everything else (ownership, streams, device
+ * errors, preconditions, results) is that of the plain call, which these
+ * forward to with the rr_dims derived from the shapes.
+ */
+#define RR_DTYPE_BF16 1
+#define RR_DTYPE_I32 2
+
+typedef struct rr_tensor {
+    void* data;
+    int32_t ndim;
+    int64_t shape[4];
+    int64_t stride[4];
+    int32_t dtype;
+} rr_tensor;
+
+int rr_kv_append_tensors(const rr_tensor* k_new, const rr_tensor* v_new, const rr_tensor* k_pool,
+                         const rr_tensor* v_pool, const rr_tensor* page_table, const rr_tensor* prefix_lens,
+                         const rr_tensor* suffix_lens, cudaStream_t stream);
+
+int rr_extend_attention_tensors(const rr_tensor* q, const rr_tensor* k_pool, const rr_tensor* v_pool,
+                                const rr_tensor* page_table, const rr_tensor* prefix_lens,
+                                const rr_tensor* suffix_lens, const rr_tensor* out, float softmax_scale,
+                                cudaStream_t stream);
 
 #ifdef __cplusplus
 }

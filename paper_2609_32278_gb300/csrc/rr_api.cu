@@ -3,6 +3,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <algorithm>
+#include <climits>
 #include <cstring>
 #include <atomic>
 #include <mutex>
@@ -789,7 +790,8 @@ constexpr size_t kNoAllocOffCu = 256;         // [0] n_units, [1] lens_ok, [2] s
 constexpr size_t kNoAllocOffUnitOff = kNoAllocOffCu + ((size_t)(kNoAllocMaxBatch + 1) * 4 + 255) / 256 * 256;
 constexpr size_t kNoAllocOffUnits = kNoAllocOffUnitOff + ((size_t)(kNoAllocMaxBatch + 1) * 4 + 255) / 256 * 256;
 constexpr size_t kNoAllocOffSlot = kNoAllocOffUnits + (size_t)kNoAllocMaxUnits * 16;
-constexpr size_t kNoAllocBytes = kNoAllocOffSlot + (size_t)kNoAllocMaxUnits * 4;  // ~1.31 MiB
+constexpr size_t kNoAllocBytes = kNoAllocOffSlot + (size_t)kNoAllocMaxUnits * 4;
+static_assert(kNoAllocBytes == 1344256, "the static scratch size stated in rr.h (1,344,256 bytes, ~1.28 MiB)");
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
 
@@ -924,4 +926,121 @@ extern "C" int rr_extend_attention_noalloc(const void* q, const void* k_pool, co
     e = rr::launch_extend_attention(a, D, (int)std::max<int64_t>(grid, 1), stream);
     if (e != cudaSuccess) return cuda_fail(e, "extend attention kernel launch");
     return RR_OK;
+}
+
+// ---------------------------------------------------------------------------
+// rr_tensor forms of the extend step's two calls: check every argument's rank, element type, shape and
+// strides on the host, derive rr_dims from the shapes and forward to the plain call.
+namespace {
+
+const char* dtype_name(int32_t d) {
+    return d == RR_DTYPE_BF16 ? "bf16" : d == RR_DTYPE_I32 ? "int32" : "unknown";
+}
+
+int check_tensor(const rr_tensor* t, const char* name, int ndim, int32_t dtype) {
+    if (!t) return fail(RR_ERR_INVALID_ARG, "%s: null rr_tensor", name);
+    if (t->ndim != ndim) return fail(RR_ERR_INVALID_ARG, "%s: %d dimensions, expected %d", name, t->ndim, ndim);
+    if (t->dtype != dtype)
+        return fail(RR_ERR_UNSUPPORTED, "%s: dtype %d (%s), expected %s", name, t->dtype, dtype_name(t->dtype),
+                    dtype_name(dtype));
+    int64_t n = 1;
+    for (int i = 0; i < ndim; ++i) {
+        if (t->shape[i] < 0) return fail(RR_ERR_INVALID_ARG, "%s: negative extent %lld in dimension %d", name,
+                                         (long long)t->shape[i], i);
+        n *= t->shape[i];
+    }
+    if (n == 0) return RR_OK;  // an empty tensor has no layout to check
+    if (!t->data) return fail(RR_ERR_INVALID_ARG, "%s: null data pointer", name);
+    int64_t expect = 1;
+    for (int i = ndim - 1; i >= 0; --i) {
+        if (t->shape[i] != 1 && t->stride[i] != expect)
+            return fail(RR_ERR_UNSUPPORTED, "%s: stride %lld in dimension %d, expected %lld (row-major contiguous)",
+                        name, (long long)t->stride[i], i, (long long)expect);
+        expect *= t->shape[i];
+    }
+    return RR_OK;
+}
+
+int same_dim(const rr_tensor* a, int ia, const char* na, const rr_tensor* b, int ib, const char* nb) {
+    if (a->shape[ia] != b->shape[ib])
+        return fail(RR_ERR_INVALID_ARG, "%s dimension %d (%lld) differs from %s dimension %d (%lld)", na, ia,
+                    (long long)a->shape[ia], nb, ib, (long long)b->shape[ib]);
+    return RR_OK;
+}
+
+int fits_i32(int64_t x, const char* what) {
+    if (x > INT32_MAX) return fail(RR_ERR_INVALID_ARG, "%s %lld exceeds int32", what, (long long)x);
+    return RR_OK;
+}
+
+// Shared checks of the pools, page table and lengths; fills every field of d except num_q_heads and
+// total_tokens.
+int check_pool_args(const rr_tensor* k_pool, const rr_tensor* v_pool, const rr_tensor* page_table,
+                    const rr_tensor* prefix_lens, const rr_tensor* suffix_lens, rr_dims* d) {
+    int rc;
+    if ((rc = check_tensor(k_pool, "k_pool", 4, RR_DTYPE_BF16))) return rc;
+    if ((rc = check_tensor(v_pool, "v_pool", 4, RR_DTYPE_BF16))) return rc;
+    for (int i = 0; i < 4; ++i)
+        if ((rc = same_dim(k_pool, i, "k_pool", v_pool, i, "v_pool"))) return rc;
+    if ((rc = check_tensor(page_table, "page_table", 2, RR_DTYPE_I32))) return rc;
+    if ((rc = check_tensor(prefix_lens, "prefix_lens", 1, RR_DTYPE_I32))) return rc;
+    if ((rc = check_tensor(suffix_lens, "suffix_lens", 1, RR_DTYPE_I32))) return rc;
+    if ((rc = same_dim(prefix_lens, 0, "prefix_lens", page_table, 0, "page_table"))) return rc;
+    if ((rc = same_dim(suffix_lens, 0, "suffix_lens", page_table, 0, "page_table"))) return rc;
+    if ((rc = fits_i32(page_table->shape[0], "batch"))) return rc;
+    if ((rc = fits_i32(page_table->shape[1], "max_pages"))) return rc;
+    if ((rc = fits_i32(k_pool->shape[1], "page_size"))) return rc;
+    if ((rc = fits_i32(k_pool->shape[2], "num_kv_heads"))) return rc;
+    if ((rc = fits_i32(k_pool->shape[3], "head_dim"))) return rc;
+    d->batch = (int32_t)page_table->shape[0];
+    d->max_pages = (int32_t)page_table->shape[1];
+    d->num_pages = k_pool->shape[0];
+    d->page_size = (int32_t)k_pool->shape[1];
+    d->num_kv_heads = (int32_t)k_pool->shape[2];
+    d->head_dim = (int32_t)k_pool->shape[3];
+    return RR_OK;
+}
+
+}  // namespace
+
+extern "C" int rr_kv_append_tensors(const rr_tensor* k_new, const rr_tensor* v_new, const rr_tensor* k_pool,
+                                    const rr_tensor* v_pool, const rr_tensor* page_table,
+                                    const rr_tensor* prefix_lens, const rr_tensor* suffix_lens,
+                                    cudaStream_t stream) {
+    g_msg[0] = 0;
+    rr_dims d{};
+    int rc;
+    if ((rc = check_pool_args(k_pool, v_pool, page_table, prefix_lens, suffix_lens, &d))) return rc;
+    if ((rc = check_tensor(k_new, "k_new", 3, RR_DTYPE_BF16))) return rc;
+    if ((rc = check_tensor(v_new, "v_new", 3, RR_DTYPE_BF16))) return rc;
+    for (int i = 0; i < 3; ++i)
+        if ((rc = same_dim(k_new, i, "k_new", v_new, i, "v_new"))) return rc;
+    if ((rc = same_dim(k_new, 1, "k_new", k_pool, 2, "k_pool"))) return rc;
+    if ((rc = same_dim(k_new, 2, "k_new", k_pool, 3, "k_pool"))) return rc;
+    d.num_q_heads = d.num_kv_heads;  // no queries in the append; any multiple of Hkv passes the dims check
+    d.total_tokens = k_new->shape[0];
+    return rr_kv_append(k_new->data, v_new->data, k_pool->data, v_pool->data,
+                        static_cast<const int32_t*>(page_table->data), static_cast<const int32_t*>(prefix_lens->data),
+                        static_cast<const int32_t*>(suffix_lens->data), &d, stream);
+}
+
+extern "C" int rr_extend_attention_tensors(const rr_tensor* q, const rr_tensor* k_pool, const rr_tensor* v_pool,
+                                           const rr_tensor* page_table, const rr_tensor* prefix_lens,
+                                           const rr_tensor* suffix_lens, const rr_tensor* out, float softmax_scale,
+                                           cudaStream_t stream) {
+    g_msg[0] = 0;
+    rr_dims d{};
+    int rc;
+    if ((rc = check_pool_args(k_pool, v_pool, page_table, prefix_lens, suffix_lens, &d))) return rc;
+    if ((rc = check_tensor(q, "q", 3, RR_DTYPE_BF16))) return rc;
+    if ((rc = check_tensor(out, "out", 3, RR_DTYPE_BF16))) return rc;
+    for (int i = 0; i < 3; ++i)
+        if ((rc = same_dim(q, i, "q", out, i, "out"))) return rc;
+    if ((rc = same_dim(q, 2, "q", k_pool, 3, "k_pool"))) return rc;
+    if ((rc = fits_i32(q->shape[1], "num_q_heads"))) return rc;
+    d.num_q_heads = (int32_t)q->shape[1];
+    d.total_tokens = q->shape[0];
+    return rr_extend_attention(q->data, k_pool->data, v_pool->data, static_cast<const int32_t*>(page_table->data),
+                               static_cast<const int32_t*>(prefix_lens->data),
+                               static_cast<const int32_t*>(suffix_lens->data), out->data, &d, softmax_scale, stream);
 }

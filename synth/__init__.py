@@ -168,16 +168,18 @@ class Workload:
 
     def manifest(self) -> Dict[str, object]:
         """What makes this batch reproducible: its name, seed and shapes, the per-agent lengths and a
-        SHA-256 of the lengths and the page table (the tensor values are a pure function of the seed and
-        the logical coordinates, so these fix every input byte)."""
+        SHA-256 over the seed, every shape field, the lengths and the page table (the tensor values are a
+        pure function of the seed and the logical coordinates, so these fix every input byte)."""
+        fields = {"seed": int(self.seed), "B": int(self.B), "Hq": int(self.Hq), "Hkv": int(self.Hkv),
+                  "D": int(self.D), "page_size": int(self.ps), "num_pages": int(self.num_pages),
+                  "max_pages": self.max_pages, "shared_len": int(self.shared_len), "T": self.T}
         h = hashlib.sha256()
+        h.update(json.dumps(fields, sort_keys=True).encode())
         for a in (self.prefix_lens, self.suffix_lens, self.page_table):
             arr = np.ascontiguousarray(a, dtype=np.int32)
             h.update(str(arr.shape).encode())
             h.update(arr.tobytes())
-        return {"name": self.name, "seed": int(self.seed), "B": int(self.B), "Hq": int(self.Hq),
-                "Hkv": int(self.Hkv), "D": int(self.D), "page_size": int(self.ps), "num_pages": int(self.num_pages),
-                "max_pages": self.max_pages, "shared_len": int(self.shared_len), "T": self.T,
+        return {"name": self.name, **fields,
                 "prefix_lens": [int(x) for x in self.prefix_lens], "suffix_lens": [int(x) for x in self.suffix_lens],
                 "sha256": h.hexdigest()}
 

@@ -77,10 +77,12 @@ def test_split_happened(rr):
     split_out = run(rr, wl, g)
     plain = torch.empty_like(g["q"])
     dims = rr.make_dims(wl.B, wl.Hq, wl.Hkv, wl.D, wl.ps, wl.max_pages, wl.num_pages, wl.T)
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
     assert fn(g["q"].data_ptr(), g["k_pool"].data_ptr(), g["v_pool"].data_ptr(), g["page_table"].data_ptr(),
               g["prefix_lens"].data_ptr(), g["suffix_lens"].data_ptr(), plain.data_ptr(), ctypes.byref(dims), 0.0,
-              None, ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)) == 0
+              err.data_ptr(), ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)) == 0
     torch.cuda.synchronize()
+    assert int(err.item()) == 0, f"device error {int(err.item())} in the allocation-free call"
     a, b = to_f64(split_out), to_f64(plain)
     assert np.abs(a - b).max() <= 2e-2
     assert not np.array_equal(bf16_bits(split_out), bf16_bits(plain))

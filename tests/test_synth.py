@@ -108,3 +108,20 @@ def test_manifest_fixes_the_inputs(tmp_path):
     h = wl.write_manifest(str(path))
     back = json.loads(path.read_text())
     assert back["sha256"] == h and back["prefix_lens"] == [16, 0] and back["suffix_lens"] == [5, 7]
+
+
+def test_manifest_hash_covers_seed_and_shapes():
+    """Batches with the same lengths and page table but another value seed or head shape hash differently."""
+    base = synth.custom("h", 2, 8, 2, 128, [64, 0], [10, 20], seed=3)
+    h0 = base.manifest()["sha256"]
+    variants = [
+        synth.Workload(**{**base.__dict__, "seed": 4}),
+        synth.Workload(**{**base.__dict__, "D": 64}),
+        synth.Workload(**{**base.__dict__, "Hq": 16}),
+        synth.Workload(**{**base.__dict__, "Hkv": 1}),
+        synth.Workload(**{**base.__dict__, "num_pages": base.num_pages + 1}),
+        synth.Workload(**{**base.__dict__, "shared_len": 16}),
+    ]
+    for v in variants:
+        assert np.array_equal(v.page_table, base.page_table)
+        assert v.manifest()["sha256"] != h0
