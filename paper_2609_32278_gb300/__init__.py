@@ -44,7 +44,11 @@ RR_ERR_SHARED = 8
 EXPORTS = ("rr_kv_append", "rr_extend_attention", "rr_extend_step", "rr_decode_attention", "rr_validate_page_table",
            "rr_get_device_error", "rr_last_error", "rr_version", "rr_shutdown", "rr_extend_attention_noalloc",
            "rr_rope_table", "rr_kv_append_rope", "rr_extend_attention_rope", "rr_extend_step_rope",
-           "rr_decode_attention_rope", "rr_decode_attention_shared", "rr_set_wait_limit")
+           "rr_decode_attention_rope", "rr_decode_attention_shared", "rr_set_wait_limit", "rr_kv_append_tensors",
+           "rr_extend_attention_tensors")
+
+RR_DTYPE_BF16 = 1
+RR_DTYPE_I32 = 2
 
 
 class RRError(RuntimeError):
@@ -57,6 +61,12 @@ class Dims(ctypes.Structure):
     _fields_ = [("batch", ctypes.c_int32), ("num_q_heads", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
                 ("head_dim", ctypes.c_int32), ("page_size", ctypes.c_int32), ("max_pages", ctypes.c_int32),
                 ("num_pages", ctypes.c_int64), ("total_tokens", ctypes.c_int64)]
+
+
+class RRTensor(ctypes.Structure):
+    """rr_tensor of include/rr.h: data pointer, rank, shape and strides (in elements), element type."""
+    _fields_ = [("data", ctypes.c_void_p), ("ndim", ctypes.c_int32), ("shape", ctypes.c_int64 * 4),
+                ("stride", ctypes.c_int64 * 4), ("dtype", ctypes.c_int32)]
 
 
 _lib = None
@@ -108,6 +118,11 @@ def lib():
         L.rr_version.argtypes = []
         L.rr_set_wait_limit.restype = None
         L.rr_set_wait_limit.argtypes = [ctypes.c_longlong]
+        tp = ctypes.POINTER(RRTensor)
+        L.rr_kv_append_tensors.restype = ctypes.c_int
+        L.rr_kv_append_tensors.argtypes = [tp] * 7 + [vp]
+        L.rr_extend_attention_tensors.restype = ctypes.c_int
+        L.rr_extend_attention_tensors.argtypes = [tp] * 7 + [ctypes.c_float, vp]
         L.rr_shutdown.restype = None
         L.rr_shutdown.argtypes = []
         _lib = L
@@ -305,6 +320,39 @@ def decode_attention(q, k_pool, v_pool, page_table, kv_lens, out=None, softmax_s
         _check(lib().rr_decode_attention(*args, _stream_ptr(stream, q.device)))
     else:
         _check(lib().rr_decode_attention_rope(*args, r[0], r[1], _stream_ptr(stream, q.device)))
+    return out
+
+
+def tensor_arg(t) -> RRTensor:
+    """The rr_tensor of a torch tensor as it is (its real strides and element type, not a checked copy), so
+    that the library's own layout checks see what the caller passes."""
+    import torch
+    codes = {torch.bfloat16: RR_DTYPE_BF16, torch.int32: RR_DTYPE_I32}
+    if t.dim() > 4:
+        raise ValueError(f"rr_tensor holds at most 4 dimensions, got {t.dim()}")
+    r = RRTensor()
+    r.data = t.data_ptr()
+    r.ndim = t.dim()
+    for i in range(t.dim()):
+        r.shape[i] = int(t.shape[i])
+        r.stride[i] = int(t.stride(i))
+    r.dtype = codes.get(t.dtype, 0)
+    return r
+
+
+def kv_append_tensors(k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens, stream=None) -> None:
+    """rr_kv_append_tensors: the append with every argument's shape, strides and type checked by the library."""
+    ts = [tensor_arg(t) for t in (k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens)]
+    _check(lib().rr_kv_append_tensors(*[ctypes.byref(t) for t in ts], _stream_ptr(stream, k_new.device)))
+
+
+def extend_attention_tensors(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, out,
+                             softmax_scale: float = 0.0, stream=None):
+    """rr_extend_attention_tensors: the attention with every argument's shape, strides and type checked by
+    the library."""
+    ts = [tensor_arg(t) for t in (q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, out)]
+    _check(lib().rr_extend_attention_tensors(*[ctypes.byref(t) for t in ts], float(softmax_scale),
+                                             _stream_ptr(stream, q.device)))
     return out
 
 
