@@ -3,10 +3,12 @@
 A step is the whole hot path for one batch of returning agents: on-device
 schedule, KV append of every uncached suffix token into its pool slot, and
 extend attention of every suffix row over its agent's cached prefix and
-suffix.  Default workload: the Llama-3-8B attention shape (32 agents, 32 query
-/ 8 KV heads, d128, page size 16, cached prefixes U[8k,32k] ending on 512-token
-chunk boundaries, suffixes U[256,2048], seeded page placement), synthetic
-N(0,1) bf16 data.
+suffix.  Default workload: the coding-agent long-context batch, the largest
+that fits one GPU (16 agents, 64 query / 8 KV heads, d128, page size 16,
+cached prefixes U[128k,256k], suffixes U[1024,4096], pages scattered over a
+pool of 90 % of free HBM), synthetic N(0,1) bf16 data.  The other long-context
+batches (Llama-3-8B shape, the LRU / RR-Evict skew pair, the shared-prefix
+batch) are timed in the same run as `configs` legs.
 
 Prints one JSON line.  `value` is the algorithmic attention TFLOP/s of the
 whole step (append included) with inputs resident in HBM; `e2e` is the same
@@ -172,12 +174,14 @@ def max_over_ranks(x, world, device=None):
     return float(t.item())
 
 
-def cpu_oracle_sample(wl, flop_budget: float, seed: int):
-    """Time the fp64 oracle on sampled suffix rows (generation of K/V is not timed)."""
+def cpu_oracle_sample(wl, flop_budget: float, seed: int, max_agents: int = 2):
+    """Time the fp64 oracle on sampled suffix rows of at most `max_agents` seeded agents (regenerating an
+    agent's K/V on the CPU, which is not timed, is what bounds the sample's wall time on long contexts)."""
     import oracle
     import synth
     rng = np.random.default_rng(seed)
     live = [b for b in range(wl.B) if wl.suffix_lens[b] > 0]
+    live = sorted(int(b) for b in rng.choice(live, size=min(max_agents, len(live)), replace=False))
     per_row = lambda b, i: 4.0 * wl.D * wl.Hq * (int(wl.prefix_lens[b]) + i + 1)
     picks, spent = {}, 0.0
     while spent < flop_budget:
@@ -206,7 +210,7 @@ def run_reference(args, world, rank):
     import synth
     if rank != 0:
         return 0
-    wl = synth.config(args.config, seed=0)
+    wl = workload(synth, args.config, seed=0)
     budget = args.ref_flops
     for _ in range(args.warmup):
         cpu_oracle_sample(wl, budget, seed=1000)
@@ -222,12 +226,12 @@ def run_reference(args, world, rank):
         "impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": tm / args.steps * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": wl.name, "inputs_sha256": wl.manifest()["sha256"][:16], "B": wl.B, "Hq": wl.Hq,
-                   "Hkv": wl.Hkv, "D": wl.D, "page_size": wl.ps,
-                   "uncached_tokens": wl.T},
+        "config": config_dict(wl, world),
+        "inputs": {"sha256": wl.manifest()["sha256"][:16], "num_pages": wl.num_pages,
+                   "note": "no pool: the oracle regenerates K/V by logical position"},
         "uncached_suffix_tokens_per_s": tok_per_s,
         "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": threads, "kind": "oracle",
-                         "sample": f"{rows} seeded suffix rows (all heads) over {args.steps} steps, "
+                         "sample": f"{rows} seeded suffix rows (all heads, 2 seeded agents per step) over {args.steps} steps, "
                                    f"~{budget:.1e} flop each; fp64 oracle, K/V generation not timed"},
         "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -236,7 +240,8 @@ def run_reference(args, world, rank):
 
 
 def load_traffic(src_hash, record="extend_attn_traffic.json"):
-    """DRAM bytes per launch from a committed ncu summary, if it was taken on this kernel source."""
+    """The committed ncu DRAM-traffic records ({workload: record}) if they were taken on this kernel source,
+    else None; and the raw file (or None)."""
     path = os.path.join(ROOT, "profiles", record)
     try:
         with open(path) as f:
@@ -245,7 +250,24 @@ def load_traffic(src_hash, record="extend_attn_traffic.json"):
         return None, None
     if rec.get("kernel_source_hash") != src_hash:
         return None, rec
-    return rec, rec
+    return rec.get("records", {}), rec
+
+
+def traffic_for(workload, src_hash, record="extend_attn_traffic.json"):
+    """DRAM bytes per launch recorded for this whole workload on this kernel source, else None."""
+    recs, _ = load_traffic(src_hash, record)
+    if not recs or workload not in recs:
+        return None
+    return recs[workload].get("dram_bytes_per_launch")
+
+
+def config_dict(wl, world):
+    """The workload as both arms name it (fields that do not depend on the pool size, which for the
+    coding-agent batch follows free HBM)."""
+    return {"workload": wl.name, "B": wl.B, "Hq": wl.Hq, "Hkv": wl.Hkv, "D": wl.D, "page_size": wl.ps,
+            "uncached_tokens": wl.T, "kv_tokens": int((wl.prefix_lens.astype(np.int64) + wl.suffix_lens).sum()),
+            "l2": f"inputs larger than L2 (KV working set {attn_bytes(wl) / 1e9:.1f} GB > 129 MB)",
+            "parallelism": f"replicas x{world}"}
 
 
 def per_agent_latency(rr, wl, g, dev, st, reps=5):
@@ -279,6 +301,67 @@ def per_agent_latency(rr, wl, g, dev, st, reps=5):
     t = np.array(times)
     return {"agents": len(times), "max_ms": float(t.max()), "p99_ms": float(np.percentile(t, 99)),
             "p50_ms": float(np.percentile(t, 50)), "mean_ms": float(t.mean()), "sum_ms": float(t.sum())}
+
+
+# The long-context batches timed beside the main workload (each as its own leg, same step, fewer steps).
+LEG_CONFIGS = (("c2_llama3_8b", 10), ("c3_lru", 5), ("c3_rr", 5), ("c5_shared", 10), ("c3g_lru", 3), ("c3g_rr", 3))
+
+
+def config_leg(rr, synth, name, steps, warmup, dev, st, peaks, rank, local):
+    """One long-context batch: append + attention steps, device-timed, with the attention's roofline and the
+    clocks seen while they ran."""
+    import torch
+    wl = workload(synth, name, seed=rank)
+    g = synth.gpu_tensors(wl, dev)
+    g["out"] = torch.empty_like(g["q"])
+
+    def append():
+        rr.kv_append(g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                     g["suffix_lens"])
+
+    def attend():
+        rr.extend_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"], g["suffix_lens"],
+                            out=g["out"])
+
+    for _ in range(warmup):
+        append()
+        attend()
+    torch.cuda.synchronize(dev)
+    if rr.device_error():
+        raise RuntimeError(f"device error in the {name} warm-up")
+    ev = [tuple(torch.cuda.Event(enable_timing=True) for _ in range(3)) for _ in range(steps)]
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    for e0, e1, e2 in ev:
+        e0.record(st)
+        append()
+        e1.record(st)
+        attend()
+        e2.record(st)
+    torch.cuda.synchronize(dev)
+    clk = clocks.stop()
+    if rr.device_error():
+        raise RuntimeError(f"device error in the {name} timed region")
+    F = attn_flops(wl)
+    step_ms = statistics.mean(e0.elapsed_time(e2) for e0, e1, e2 in ev)
+    attn_ms = statistics.mean(e1.elapsed_time(e2) for e0, e1, e2 in ev)
+    app_ms = statistics.mean(e0.elapsed_time(e1) for e0, e1, e2 in ev)
+    achieved = F / (attn_ms * 1e-3) / 1e12
+    res = {"config": config_dict(wl, 1), "inputs_sha256": wl.manifest()["sha256"][:16], "steps": steps,
+           "warmup": warmup, "ms_per_step": step_ms, "value": F / (step_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
+           "uncached_suffix_tokens_per_s": wl.T / (step_ms * 1e-3), "attention_ms": attn_ms,
+           "attention_ms_median": statistics.median(e1.elapsed_time(e2) for e0, e1, e2 in ev),
+           "kv_append_ms": app_ms, "kv_append_gbs": append_bytes(wl) / (app_ms * 1e-3) / 1e9,
+           "roofline": {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16"], "unit": "TFLOP/s",
+                        "frac": achieved / peaks["bf16"], "frac_of_sustained": achieved / peaks["bf16_sus"],
+                        "frac_of_nominal": achieved / NOMINAL_BF16_TFLOPS,
+                        "traffic": traffic_for(wl.name, kernel_source_hash()),
+                        "algorithmic_flops": F, "algorithmic_bytes": attn_bytes(wl)},
+           "clocks": clk}
+    del g
+    torch.cuda.empty_cache()
+    return res
 
 
 def decode_bytes(wl) -> float:
@@ -322,8 +405,7 @@ def decode_leg(args, rr, synth, dev, st, peaks, rank):
     nbytes = decode_bytes(wl)
     gbs = nbytes / (ms * 1e-3) / 1e9
     dec_hash = kernel_source_hash(DECODE_SOURCES)
-    rec, _ = load_traffic(dec_hash, "decode_attn_traffic.json")
-    traffic = rec.get("dram_bytes_per_launch") if rec is not None and rec.get("workload") == wl.name else None
+    traffic = traffic_for(wl.name, dec_hash, "decode_attn_traffic.json")
     res = {"workload": wl.name, "inputs_sha256": wl.manifest()["sha256"][:16], "B": wl.B, "Hq": wl.Hq,
            "Hkv": wl.Hkv, "D": wl.D,
            "kv_tokens": int((wl.prefix_lens.astype(np.int64) + 1).sum()), "calls": n, "ms_per_call": ms,
@@ -362,8 +444,9 @@ def decode_leg(args, rr, synth, dev, st, peaks, rank):
     return res
 
 
-# Replay leg: the policy's effect on per-request extend cost (Sec. 4's P99 metrics), with the attention
-# time of each request taken from a cost model fitted to this GPU's measured extend kernel.
+# Replay leg: the policy's effect on per-request extend cost (Sec. 4's P99 metrics).  Every extend batch a
+# policy's replay produces is run through rr_kv_append + rr_extend_attention on this GPU and timed with CUDA
+# events; a request's attention time to first token is its batch's time (one layer).
 REPLAY_MODELS = {  # attention geometry of the two served models of Sec. 4
     "conversational": {"model": "Qwen3-Coder-30B-A3B attention (32 q / 4 kv heads, d128)", "Hq": 32, "Hkv": 4},
     "coding": {"model": "Qwen3-8B attention (32 q / 8 kv heads, d128)", "Hq": 32, "Hkv": 8},
@@ -372,62 +455,67 @@ REPLAY_MODELS = {  # attention geometry of the two served models of Sec. 4
 # points inside the regime of Eq. 1 on these traces (active demand fits, live idle demand does not) --
 # at 0.6 and above nothing is evicted from live agents, far below it every policy thrashes
 REPLAY_SETTINGS = [
-    ("conversational", 222, 40, 0.4), ("conversational", 222, 80, 0.4), ("conversational", 222, 80, 0.6),
-    ("coding", 64, 16, 0.4), ("coding", 64, 16, 0.5), ("coding", 64, 32, 0.4),
+    ("conversational", 222, 40, 0.4), ("conversational", 222, 80, 0.4), ("coding", 64, 16, 0.5),
+    ("coding", 64, 16, 0.4),
 ]
 REPLAY_POLICIES = [  # label, policy, completion signals
     ("lru", "lru", False), ("lru+cs", "lru", True), ("rr-evict+cs", "rr", True), ("rr-tiered", "tiered", False),
 ]
+REPLAY_WINDOW_S = 0.05  # requests arriving within one 50 ms scheduling tick share an extend batch
 
 
-def measure_extend_grid(rr, synth, dev, st, Hq, Hkv, D=128, reps=5):
-    """Median CUDA-event time of one agent's append + extend attention for a grid of (P, S)."""
+def measure_batches(rr, synth, dev, st, batches, Hq, Hkv, D=128, ps=16):
+    """CUDA-event time (seconds) of append + extend attention for each (prefix_lens, suffix_lens) batch.
+
+    One pool holds the largest batch: agent i of a batch takes the next distinct pages of a seeded
+    placement, every one of them filled with the generator's values; q / k_new / v_new are the first T rows
+    of one generated buffer.  Each batch runs once untimed, then once timed."""
     import torch
-    out = []
-    for P in (0, 2048, 8192, 32768, 131072):
-        for S in (64, 256, 1024, 4096, 16384, 65536, 131072):
-            if P + S > 262144:
-                continue
-            wl = synth.custom(f"grid_{P}_{S}", 1, Hq, Hkv, D, [P], [S], seed=11)
-            g = synth.gpu_tensors(wl, dev)
-            args = (g["q"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"], g["suffix_lens"])
-            o = torch.empty_like(g["q"])
-            for _ in range(2):
-                rr.kv_append(g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
-                             g["suffix_lens"])
-                rr.extend_attention(*args, out=o)
-            ts = []
-            for _ in range(reps):
-                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    need = max(sum(-(-(int(p) + int(s)) // ps) for p, s in zip(P, S)) for P, S in batches)
+    t_max = max(sum(int(s) for s in S) for P, S in batches)
+    pool = synth.custom("replay_pool", 1, Hq, Hkv, D, [need * ps], [0], ps=ps, seed=13)
+    rows = synth.custom("replay_rows", 1, Hq, Hkv, D, [0], [t_max], ps=ps, seed=14)
+    gp = synth.gpu_tensors(pool, dev)
+    gr = synth.gpu_tensors(rows, dev)
+    pages = pool.page_table[0]
+    out = torch.empty_like(gr["q"])
+    times = []
+    for P, S in batches:
+        B = len(P)
+        pb = [-(-(int(p) + int(s)) // ps) for p, s in zip(P, S)]
+        pt = np.full((B, max(pb)), -1, dtype=np.int32)
+        off = 0
+        for i, n in enumerate(pb):
+            pt[i, :n] = pages[off:off + n]
+            off += n
+        T = int(sum(S))
+        a = (torch.from_numpy(pt).to(dev), torch.tensor(np.asarray(P, dtype=np.int32), device=dev),
+             torch.tensor(np.asarray(S, dtype=np.int32), device=dev))
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        for k in range(2):
+            if k:
                 e0.record(st)
-                rr.kv_append(g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
-                             g["suffix_lens"])
-                rr.extend_attention(*args, out=o)
-                e1.record(st)
-                e1.synchronize()
-                ts.append(e0.elapsed_time(e1) * 1e-3)
-            if rr.device_error():
-                raise RuntimeError("device error in the replay cost grid")
-            out.append((P, S, statistics.median(ts)))
-            del g, o
+            rr.kv_append(gr["k_new"][:T], gr["v_new"][:T], gp["k_pool"], gp["v_pool"], *a)
+            rr.extend_attention(gr["q"][:T], gp["k_pool"], gp["v_pool"], *a, out=out[:T])
+        e1.record(st)
+        e1.synchronize()
+        times.append(e0.elapsed_time(e1) * 1e-3)
+    if rr.device_error():
+        raise RuntimeError("device error in the replay batches")
+    del gp, gr, out
     torch.cuda.empty_cache()
-    return out
+    return times
 
 
 def replay_leg(rr, synth, dev, st):
     from paper_2609_32278_gb300 import policy as pol
-    res = {"note": ("synthetic agent traces (policy.synthetic_traces) replayed under each policy; attention "
-                    "time per request = c0 + c1 S + c2 F(P, S) + c3 (P + S) fitted to this GPU's measured "
-                    "single-agent append + extend time (one layer)"), "models": {}, "runs": []}
-    costs = {}
-    for kind, m in REPLAY_MODELS.items():
-        grid = measure_extend_grid(rr, synth, dev, st, m["Hq"], m["Hkv"])
-        cost, coef, rel = pol.fit_extend_cost(grid, m["Hq"], 128)
-        costs[kind] = cost
-        res["models"][kind] = {"model": m["model"], "coef_s_call_token_flop_key": coef,
-                               "fit_max_rel_err": rel, "grid_points": len(grid),
-                               "grid": [(P, S, round(t * 1e3, 4)) for P, S, t in grid]}
+    res = {"note": ("synthetic agent traces (policy.synthetic_traces) replayed under each policy; each extend "
+                    f"batch (requests within {REPLAY_WINDOW_S * 1e3:.0f} ms) run through rr_kv_append + "
+                    "rr_extend_attention on this GPU and timed with CUDA events (one layer); a request's "
+                    "attention time is its batch's"), "models": {k: m["model"] for k, m in REPLAY_MODELS.items()},
+           "runs": []}
     for kind, n, conc, frac in REPLAY_SETTINGS:
+        m = REPLAY_MODELS[kind]
         traces = pol.synthetic_traces(n, kind, seed=0)
         finals = sorted(sum(t.new_tokens) + sum(t.output_tokens) for t in traces)
         cap = int(frac * sum(finals[-conc:]))
@@ -436,9 +524,54 @@ def replay_leg(rr, synth, dev, st):
         for label, policy, cs in REPLAY_POLICIES:
             reqs = pol.replay(traces, cap, policy, shared_prompt=2048, chunk=1024, completion_signals=cs,
                               concurrency=conc)
-            run["policies"][label] = pol.summarize(reqs, costs[kind])
+            batches = pol.extend_batches(reqs, REPLAY_WINDOW_S)
+            bt = measure_batches(rr, synth, dev, st, [(P, S) for _, P, S in batches], m["Hq"], m["Hkv"])
+            per_req = [0.0] * len(reqs)
+            for (idx, _, _), t in zip(batches, bt):
+                for i in idx:
+                    per_req[i] = t
+            summ = pol.summarize(reqs, per_req)
+            sizes = [len(idx) for idx, _, _ in batches]
+            summ.update({"batches": len(batches), "batch_size_max": max(sizes), "batch_size_mean": float(np.mean(sizes)),
+                         "batch_ms_p50": 1e3 * pol.percentile(bt, 50), "batch_ms_p99": 1e3 * pol.percentile(bt, 99),
+                         "batch_ms_max": 1e3 * max(bt), "gpu_s_total": float(sum(bt))})
+            run["policies"][label] = summ
         res["runs"].append(run)
     return res
+
+
+# The LRU / RR-Evict skew pair drawn from the eviction-policy generator rather than from length samplers:
+# 64 coding agents (Qwen3-8B attention: 32 q / 8 kv heads, d128) all admitted, a cache of half their summed
+# final contexts, and the batch in which every agent returns with its next request after the median request
+# time (policy.snapshot_lengths); the 2048-token system prompt stays shared.
+POLICY_PAIR = {"c3g_lru": ("lru", False), "c3g_rr": ("rr", True)}
+
+
+def policy_workload(synth, name, seed=0):
+    from paper_2609_32278_gb300 import policy as pol
+    policy, cs = POLICY_PAIR[name]
+    traces = pol.synthetic_traces(64, "coding", seed=seed)
+    cap = int(0.5 * sum(sum(t.new_tokens) + sum(t.output_tokens) for t in traces))
+    reqs = pol.replay(traces, cap, policy, shared_prompt=2048, chunk=1024, completion_signals=cs, concurrency=64)
+    P, S = pol.snapshot_lengths(reqs, 0.5)
+    return synth.custom(name, len(P), 32, 8, 128, P, S, shared_len=2048, seed=seed)
+
+
+def workload(synth, name, seed=0, free_hbm_bytes=None):
+    if name in POLICY_PAIR:
+        return policy_workload(synth, name, seed)
+    return synth.config(name, seed=seed, free_hbm_bytes=free_hbm_bytes)
+
+
+def slice_workload(synth, wl, agents=0, stride=1):
+    """A small profiling case: every `stride`-th agent of `wl` (a systematic sample keeps the batch's mix of
+    agent kinds), the first `agents` of those if nonzero, in a pool of twice the pages they need."""
+    idx = np.arange(0, wl.B, max(1, stride))
+    if agents:
+        idx = idx[:agents]
+    name = wl.name + (f"[::{stride}]" if stride > 1 else "") + (f"[:{agents}]" if agents else "")
+    return synth.custom(name, len(idx), wl.Hq, wl.Hkv, wl.D, wl.prefix_lens[idx], wl.suffix_lens[idx], ps=wl.ps,
+                        shared_len=wl.shared_len, seed=wl.seed)
 
 
 def run_ours(args, world, rank, local):
@@ -449,11 +582,9 @@ def run_ours(args, world, rank, local):
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     free = torch.cuda.mem_get_info(dev)[0]
-    wl = synth.config(args.config, seed=rank, free_hbm_bytes=free if args.config == "c4_coding" else None)
-    if args.agents:
-        wl = synth.custom(f"{args.config}[:{args.agents}]", args.agents, wl.Hq, wl.Hkv, wl.D,
-                          wl.prefix_lens[:args.agents], wl.suffix_lens[:args.agents], ps=wl.ps,
-                          shared_len=wl.shared_len, seed=wl.seed)
+    wl = workload(synth, args.config, seed=rank, free_hbm_bytes=free if args.config == "c4_coding" else None)
+    if args.agents or args.agent_stride > 1:
+        wl = slice_workload(synth, wl, args.agents, args.agent_stride)
     g = synth.gpu_tensors(wl, dev)
     st = torch.cuda.current_stream(dev)
     F = attn_flops(wl)
@@ -636,23 +767,22 @@ def run_ours(args, world, rank, local):
     per_agent = None
     if args.per_agent:
         per_agent = per_agent_latency(rr, wl, g, dev, st)
+    g.clear()
+    torch.cuda.empty_cache()
     replay = None
     if args.replay and rank == 0:
-        g.clear()
-        torch.cuda.empty_cache()
         replay = replay_leg(rr, synth, dev, st)
+    legs = None
+    if not args.no_legs:
+        legs = [config_leg(rr, synth, name, min(args.steps, n), args.warmup, dev, st, peaks, rank, local)
+                for name, n in LEG_CONFIGS if name != args.config]
     decode = None
     if not args.no_decode:
-        g.clear()
-        torch.cuda.empty_cache()
         decode = decode_leg(args, rr, synth, dev, st, peaks, rank)
 
     achieved = F / (attn_ms * 1e-3) / 1e12
     src_hash = kernel_source_hash()
-    traffic_rec, _ = load_traffic(src_hash)
-    traffic = None
-    if traffic_rec is not None and traffic_rec.get("workload") == wl.name:  # the whole batch it was captured on, not a slice
-        traffic = traffic_rec.get("dram_bytes_per_launch")
+    traffic = traffic_for(wl.name, src_hash)  # recorded for this whole batch (scaled from a slice), or None
     roof = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16"], "unit": "TFLOP/s",
             "frac": achieved / peaks["bf16"], "traffic": traffic,
             "peak_kind": f"{peaks['src']} bf16 dense burst (the timed loop is well under a second)",
@@ -666,11 +796,9 @@ def run_ours(args, world, rank, local):
         "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": wl.name, "inputs_sha256": wl.manifest()["sha256"][:16], "B": wl.B, "Hq": wl.Hq,
-                   "Hkv": wl.Hkv, "D": wl.D, "page_size": wl.ps,
-                   "uncached_tokens": wl.T, "kv_tokens": int((wl.prefix_lens + wl.suffix_lens).sum()),
-                   "num_pages": wl.num_pages, "l2": "inputs larger than L2 (KV working set "
-                   f"{attn_bytes(wl) / 1e9:.1f} GB > 129 MB)", "parallelism": f"replicas x{world}"},
+        "config": config_dict(wl, world),
+        "inputs": {"sha256": wl.manifest()["sha256"][:16], "num_pages": wl.num_pages,
+                   "pool_gb": 2.0 * wl.num_pages * wl.ps * wl.Hkv * wl.D * 2 / 1e9},
         "uncached_suffix_tokens_per_s": tok_s,
         "attention_ms": attn_ms, "kv_append_ms": app_ms,
         "attention_ms_median": statistics.median(ev[k][1].elapsed_time(ev[k][2]) for k in range(args.steps)),
@@ -687,6 +815,8 @@ def run_ours(args, world, rank, local):
         line["fused_step"] = fused
     if rope is not None:
         line["rope_step"] = rope
+    if legs is not None:
+        line["configs"] = legs
     if decode is not None:
         line["decode"] = decode
     if replay is not None:
@@ -694,7 +824,7 @@ def run_ours(args, world, rank, local):
     if rank == 0 and not args.no_cpu_baseline:
         f, t, rows, threads = cpu_oracle_sample(wl, args.baseline_flops, seed=7)
         line["cpu_baseline"] = {"value": f / t / 1e12, "unit": "TFLOP/s", "cores": threads, "kind": "oracle",
-                                "sample": f"{rows} seeded suffix rows (all {wl.Hq} heads) of {args.config}, "
+                                "sample": f"{rows} seeded suffix rows (all {wl.Hq} heads) of 2 seeded agents of {args.config}, "
                                           f"{f:.2e} flop; fp64 oracle; K/V generation not timed"}
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -707,11 +837,14 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    ap.add_argument("--config", default="c2_llama3_8b")
+    ap.add_argument("--config", default="c4_coding")
+    ap.add_argument("--no-legs", action="store_true", help="skip the other long-context batches' legs")
     ap.add_argument("--ref-flops", type=float, default=1e10, help="oracle flops per reference-arm step")
     ap.add_argument("--baseline-flops", type=float, default=3e11, help="oracle flops of the cpu_baseline sample (~10 s on 16 cores)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--agents", type=int, default=0, help="only the first N agents (small profiling case)")
+    ap.add_argument("--agent-stride", type=int, default=1,
+                    help="only every K-th agent (small profiling case with the batch's mix of agent kinds)")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
     ap.add_argument("--per-agent", action="store_true", help="also time each agent's extend step alone")
     ap.add_argument("--decode-config", default="c2_decode", help="decode batch of the decode leg")
@@ -720,7 +853,7 @@ def main():
     ap.add_argument("--no-rope", action="store_true", help="skip the rotary-embedding step leg")
     ap.add_argument("--decode-agents", type=int, default=0, help="only the first N agents of the decode batch")
     ap.add_argument("--replay", action="store_true",
-                    help="also replay synthetic agent traces under each eviction policy (modelled attention TTFT)")
+                    help="also replay synthetic agent traces under each eviction policy, timing every extend batch")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -47,11 +47,46 @@ def test_record_taken_only_for_its_hash(tmp_path, monkeypatch):
     _tree(tmp_path)
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
     h = bench.kernel_source_hash()
-    rec = {"kernel_source_hash": h, "workload": "c2_llama3_8b", "dram_bytes_per_launch": 123}
+    recs = {"c4_coding": {"dram_bytes_per_launch": 123, "slice": "c4_coding[:2]"},
+            "c4_coding[:2]": {"dram_bytes_per_launch": 17}}
+    rec = {"kernel_source_hash": h, "records": recs}
     (tmp_path / "profiles" / "extend_attn_traffic.json").write_text(json.dumps(rec))
     got, raw = bench.load_traffic(h)
-    assert got == rec and raw == rec
+    assert got == recs and raw == rec
+    assert bench.traffic_for("c4_coding", h) == 123
+    assert bench.traffic_for("c4_coding[:2]", h) == 17
+    assert bench.traffic_for("c2_llama3_8b", h) is None                        # not recorded
     got, raw = bench.load_traffic("0" * 16)
     assert got is None and raw == rec
+    assert bench.traffic_for("c4_coding", "0" * 16) is None                   # recorded on other code
     assert bench.load_traffic(h, "decode_attn_traffic.json") == (None, None)   # no such record
 
+
+def test_both_arms_name_the_same_config():
+    """The reference arm builds the coding-agent batch without a GPU (pool size unknown); the config both
+    arms report leaves the pool size out, so it is the same."""
+    import synth
+    a = synth.config("c4_coding", seed=0, free_hbm_bytes=250 * 2 ** 30)
+    b = synth.config("c4_coding", seed=0)
+    assert a.num_pages != b.num_pages
+    assert bench.config_dict(a, 1) == bench.config_dict(b, 1)
+
+
+
+def test_policy_pair_workloads():
+    """The generator-drawn skew pair (bench legs c3g_lru / c3g_rr): same agents, the shared system prompt on
+    common pages, whole-history recomputes under LRU against short tails under RR-Evict, valid page tables."""
+    import numpy as np
+    import synth
+    a = bench.workload(synth, "c3g_lru")
+    b = bench.workload(synth, "c3g_rr")
+    assert a.B == b.B > 32 and a.shared_len == b.shared_len == 2048
+    assert (a.Hq, a.Hkv, a.D) == (b.Hq, b.Hkv, b.D) == (32, 8, 128)
+    assert a.suffix_lens.max() > 8 * b.suffix_lens.max()
+    assert np.all(a.prefix_lens >= 2048) and np.all(b.prefix_lens >= 2048)
+    # every agent's first 128 logical pages are the shared ones
+    assert np.all(a.page_table[:, :128] == a.page_table[0, :128])
+    import paper_2609_32278_gb300 as rr
+    if os.path.exists(rr._SO):
+        for w in (a, b):
+            assert rr.validate_page_table(w.page_table, w.prefix_lens, w.suffix_lens, w.num_pages, w.ps) == 0
