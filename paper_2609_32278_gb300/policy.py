@@ -457,46 +457,48 @@ def percentile(values, p: float) -> float:
     return float(v[k])
 
 
-def summarize(requests: List[Request], cost=None) -> Dict[str, float]:
-    """Sec. 4's per-request metrics: uncached prompt tokens (P50, P99, mean, max) and, given
-    cost(P, S) -> seconds, the modelled attention time of each request's extend (P50, P99, mean, max)."""
+def summarize(requests: List[Request], times=None) -> Dict[str, float]:
+    """Sec. 4's per-request metrics: uncached prompt tokens (P50, P99, mean, max) and, given each request's
+    measured extend time in seconds (`times[i]` for requests[i]; 0 for a request with nothing to extend),
+    the attention part of its time to first token (P50, P99, mean, max)."""
     unc = [r.uncached for r in requests]
     res = {"requests": len(requests), "uncached_p50": percentile(unc, 50), "uncached_p99": percentile(unc, 99),
            "uncached_mean": sum(unc) / len(unc), "uncached_max": float(max(unc))}
-    if cost is not None:
-        t = [cost(r.cached, r.uncached) for r in requests]
+    if times is not None:
+        t = list(times)
         res.update({"ttft_attn_p50_ms": 1e3 * percentile(t, 50), "ttft_attn_p99_ms": 1e3 * percentile(t, 99),
                     "ttft_attn_mean_ms": 1e3 * sum(t) / len(t), "ttft_attn_max_ms": 1e3 * max(t)})
     return res
 
 
-def fit_extend_cost(samples, Hq: int, D: int):
-    """Least-squares fit of t(P, S) = c0 + c1 S + c2 F(P, S) + c3 (P + S) to measured (P, S, seconds) samples,
-    weighted by 1/t (relative error).  F = 4 D Hq (S P + S (S + 1) / 2) is the extend attention's flops
-    (the tensor-bound part); P + S, the keys read, carries what flops miss when a short suffix over a long
-    prefix leaves few work units in flight.  Coefficients are clipped at zero.  Returns (cost function,
-    (c0, c1, c2, c3), max relative error over the samples)."""
-    import numpy as np
-
-    def feats(P, S):
-        return [1.0, float(S), 4.0 * D * Hq * (S * P + S * (S + 1) / 2.0), float(P + S)]
-
-    A = np.asarray([feats(P, S) for P, S, _ in samples])
-    y = np.asarray([t for _, _, t in samples])
-    w = 1.0 / y
-    coef, *_ = np.linalg.lstsq(A * w[:, None], y * w, rcond=None)
-    coef = np.maximum(coef, 0.0)
-
-    def cost(P, S):
-        if S <= 0:
-            return 0.0
-        return float(np.dot(coef, feats(P, S)))
-
-    rel = float(np.max(np.abs(A @ coef - y) / y))
-    return cost, tuple(float(c) for c in coef), rel
+def extend_batches(requests: List[Request], window: float = 0.05):
+    """The extend batches a prefill engine launches: requests in arrival order, each batch taking every
+    request that arrives within `window` seconds of its first one (one scheduling tick).  Returns a list of
+    (request indices, prefix_lens, suffix_lens); requests with nothing uncached are left out (no extend)."""
+    order = sorted((i for i, r in enumerate(requests) if r.uncached > 0), key=lambda i: (requests[i].time, i))
+    out = []
+    k = 0
+    while k < len(order):
+        t0 = requests[order[k]].time
+        j = k
+        while j < len(order) and requests[order[j]].time - t0 <= window:
+            j += 1
+        idx = order[k:j]
+        out.append((idx, [requests[i].cached for i in idx], [requests[i].uncached for i in idx]))
+        k = j
+    return out
 
 
-def batch_lengths(requests: List[Request], batch: int, start: int = 0):
-    """(prefix_lens, suffix_lens) of `batch` consecutive requests: the extend batch they form."""
-    sel = requests[start:start + batch]
-    return [r.cached for r in sel], [r.uncached for r in sel]
+def snapshot_lengths(requests: List[Request], quantile: float = 0.5):
+    """(prefix_lens, suffix_lens) of the batch in which every agent returns at once: each agent's first
+    request at or after the time by which `quantile` of all requests have arrived, in agent order.  The
+    cached prefixes are what the policy left each agent at that moment, so the batch has the policy's
+    (P, S) distribution (Sec. 3.3, Eq. 3)."""
+    times = sorted(r.time for r in requests)
+    t_star = times[min(len(times) - 1, int(len(times) * quantile))]
+    first: Dict[int, Request] = {}
+    for r in sorted(requests, key=lambda r: (r.time, r.agent)):
+        if r.time >= t_star and r.agent not in first:
+            first[r.agent] = r
+    agents = sorted(first)
+    return [first[a].cached for a in agents], [first[a].uncached for a in agents]

@@ -1,8 +1,10 @@
-"""Parity at the five workloads' full sizes, in the launch configuration bench.py times.
+"""Parity at the five workloads' full sizes, and on the LRU / RR-Evict pair drawn from the eviction-policy
+generator, in the launch configuration bench.py times.
 
-Attention: seeded sample of suffix rows (every agent's first and last row, a
-window of consecutive rows covering two whole Q tiles of the agent with the
-longest prefix, random rows up to an fp64 flop budget), all heads of each,
+Attention: seeded sample of suffix rows (every sampled agent's first and last
+row, a window of consecutive rows covering two whole Q tiles of the agent with
+the longest prefix -- of each of 8 sampled agents on c4, whose key ranges are
+the deepest -- and random rows up to an fp64 flop budget), all heads of each,
 against the oracle computed from logically generated K/V -- never from the
 GPU pool, so a page-indexing mistake cannot cancel out.
 
@@ -11,6 +13,8 @@ k_new / v_new row bit for bit; every other slot of the pool keeps its content
 (per-slot checksums before and after).
 """
 import math
+import os
+import sys
 
 import numpy as np
 import pytest
@@ -18,9 +22,12 @@ import pytest
 import synth
 from parity import check_close, oracle_sampled, sample_rows, to_f64
 
+sys.path.insert(0, os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
+import bench  # noqa: E402  (the workload definitions bench.py times)
+
 pytestmark = pytest.mark.gpu
 
-CONFIGS = ["c2_llama3_8b", "c3_lru", "c3_rr", "c5_shared", "c4_coding"]
+CONFIGS = ["c2_llama3_8b", "c3_lru", "c3_rr", "c5_shared", "c4_coding", "c3g_lru", "c3g_rr"]
 
 
 @pytest.fixture(scope="module")
@@ -56,7 +63,7 @@ def test_full_size_config(rr, name):
     import torch
     torch.cuda.empty_cache()
     free = torch.cuda.mem_get_info()[0]
-    wl = synth.config(name, free_hbm_bytes=free if name == "c4_coding" else None)
+    wl = bench.workload(synth, name, free_hbm_bytes=free if name == "c4_coding" else None)
     g = synth.gpu_tensors(wl, "cuda")
     before_k = _slot_checksums(g["k_pool"])
     before_v = _slot_checksums(g["v_pool"])
@@ -81,7 +88,9 @@ def test_full_size_config(rr, name):
     del before_k, before_v, mask
 
     # ---- attention: sampled rows vs the oracle
-    rows = sample_rows(wl, flop_budget=2.5e11, seed=1, max_agents=5 if name == "c4_coding" else 12)
+    # c4 has the deepest key ranges (128k-256k): 8 agents, each with a whole work unit of consecutive rows
+    deep = name == "c4_coding"
+    rows = sample_rows(wl, flop_budget=2.5e11, seed=1, max_agents=8 if deep else 12, window_every_agent=deep)
     ref = oracle_sampled(wl, rows, 1.0 / math.sqrt(wl.D))
     cu = wl.cu
     got_rows, ref_rows = [], []
@@ -91,7 +100,7 @@ def test_full_size_config(rr, name):
         ref_rows.append(ref[b])
     stats = check_close(np.concatenate(got_rows), np.concatenate(ref_rows), name)
     n_rows = sum(len(r) for r in rows.values())
-    print(f"{name}: {n_rows} rows x {wl.Hq} heads checked, max {stats['max']:.2e} mean {stats['mean']:.2e} "
-          f"p99.9 {stats['p999']:.2e}")
+    print(f"{name}: {n_rows} rows of {len(rows)} agents x {wl.Hq} heads checked ({stats['n']} elements in the "
+          f"mean), max {stats['max']:.2e} mean {stats['mean']:.2e} p99.9 {stats['p999']:.2e}")
     del g, out
     torch.cuda.empty_cache()

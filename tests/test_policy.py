@@ -222,21 +222,50 @@ def test_percentile_is_nearest_rank():
     assert pol.percentile([5], 99) == 5 and pol.percentile([3, 1, 2], 0) == 1
 
 
-def test_fit_extend_cost_recovers_a_known_model():
-    c0, c1, c2, c3 = 2e-5, 3e-9, 1.0 / 1.3e15, 4e-9
-    model = lambda P, S: c0 + c1 * S + c2 * 4.0 * 128 * 32 * (S * P + S * (S + 1) / 2.0) + c3 * (P + S)
-    samples = [(P, S, model(P, S)) for P in (0, 1000, 8000, 64000) for S in (64, 512, 4096, 32000)]
-    cost, coef, rel = pol.fit_extend_cost(samples, 32, 128)
-    assert rel < 1e-6
-    assert coef[0] == pytest.approx(c0, rel=1e-4) and coef[2] == pytest.approx(c2, rel=1e-6)
-    assert coef[3] == pytest.approx(c3, rel=1e-4)
-    assert cost(1000, 512) == pytest.approx(model(1000, 512))
-    assert cost(500, 0) == 0.0
+def test_extend_batches_group_by_arrival_window():
+    def req(agent, t, cached, uncached):
+        return pol.Request(agent, 0, t, cached + uncached, cached)
+
+    reqs = [req(0, 0.00, 60, 40), req(1, 0.03, 0, 50), req(2, 0.06, 60, 10), req(3, 0.04, 0, 90),
+            req(4, 0.20, 30, 0), req(5, 0.21, 55, 5)]
+    got = pol.extend_batches(reqs, window=0.05)
+    # [0.00, 0.05]: requests 0, 1, 3 (in arrival order); then 2 alone; 4 has nothing uncached; then 5
+    assert [b[0] for b in got] == [[0, 1, 3], [2], [5]]
+    assert got[0][1] == [60, 0, 0] and got[0][2] == [40, 50, 90]
+    assert got[2][1] == [55] and got[2][2] == [5]
+    flat = sorted(i for b in got for i in b[0])
+    assert flat == [i for i, r in enumerate(reqs) if r.uncached > 0]
+
+
+def test_snapshot_lengths_take_each_agents_next_request():
+    # Request(agent, turn, time, prompt_len, cached)
+    reqs = [pol.Request(0, 0, 0.0, 100, 0), pol.Request(1, 0, 1.0, 200, 0), pol.Request(0, 1, 2.0, 300, 150),
+            pol.Request(1, 1, 3.0, 400, 20), pol.Request(0, 2, 4.0, 500, 500), pol.Request(1, 2, 5.0, 600, 90)]
+    # the median request arrives at t = 3.0: agent 0's next is its turn 2, agent 1's its turn 1
+    P, S = pol.snapshot_lengths(reqs, 0.5)
+    assert P == [500, 20] and S == [0, 380]
+
+
+def test_snapshot_pair_shows_the_two_recompute_shapes():
+    """The generator-drawn skew pair: under LRU a few agents recompute their whole history (long suffixes
+    over the shared prompt alone), under RR-Evict every agent recomputes a shorter tail (Eq. 3)."""
+    traces = pol.synthetic_traces(64, "coding", seed=0)
+    finals = sorted(sum(t.new_tokens) + sum(t.output_tokens) for t in traces)
+    cap = int(0.5 * sum(finals))
+    res = {}
+    for label, policy, cs in (("lru", "lru", False), ("rr", "rr", True)):
+        reqs = pol.replay(traces, cap, policy, shared_prompt=2048, chunk=1024, completion_signals=cs,
+                          concurrency=64)
+        res[label] = pol.snapshot_lengths(reqs, 0.5)
+    (Pl, Sl), (Pr, Sr) = res["lru"], res["rr"]
+    assert len(Sl) == len(Sr) > 32
+    assert max(Sl) > 8 * max(Sr) and sum(Sl) > sum(Sr)
+    assert min(Pl) == 2048 and min(Pr) >= 2048   # the shared system prompt is never evicted
 
 
 def test_summarize_reports_the_sec4_metrics():
     reqs = [pol.Request(0, k, float(k), 100 + k, 100 - k) for k in range(50)]
-    s = pol.summarize(reqs, cost=lambda P, S: 1e-3 * S)
+    s = pol.summarize(reqs, times=[1e-3 * r.uncached for r in reqs])
     assert s["requests"] == 50 and s["uncached_max"] == 2 * 49
     assert s["uncached_p99"] == pol.percentile([2 * k for k in range(50)], 99)
     assert s["ttft_attn_max_ms"] == pytest.approx(98.0)
