@@ -124,6 +124,11 @@ int rr_extend_attention(const void* q, const void* k_pool, const void* v_pool, c
  * into the pool slots page_table assigns to them, for later calls.  Arguments,
  * layouts, preconditions and errors are those of the two calls it replaces;
  * k_pool / v_pool are written, so they are non-const here.
+ *
+ * Performance: it launches two kernels where the two calls launch four, which
+ * makes it faster for a small extend (one agent, a few thousand keys: ~1.1x
+ * measured on GB300), and slower for large batches (~0.9x), where the
+ * separate append pass it saves is well under 1 % of the step.
  */
 int rr_extend_step(const void* q, const void* k_new, const void* v_new, void* k_pool, void* v_pool,
                    const int32_t* page_table, const int32_t* prefix_lens, const int32_t* suffix_lens, void* out,
