@@ -36,11 +36,22 @@ __device__ __forceinline__ int last_le(const int32_t* off, int n, long long x) {
 }
 
 constexpr int kAppendThreads = 256;
+constexpr int kCuSmem = 2048;  // agents whose suffix prefix sums a block stages in shared memory
+
 
 template <bool kRope>
 __global__ void __launch_bounds__(kAppendThreads) kv_append_kernel(const AppendArgs a) {
+    __shared__ int32_t s_cu[kCuSmem];
     ptx::griddep_wait();  // the schedule kernel's output (launched as its dependent)
     if (*a.lens_ok == 0) return;
+    // each token's agent is a binary search over the suffix prefix sums: from shared memory when they fit,
+    // so a token's copy does not wait behind log2(B) dependent global loads
+    const bool cu_in_smem = a.B < kCuSmem;
+    if (cu_in_smem) {
+        for (int i = threadIdx.x; i <= a.B; i += kAppendThreads) s_cu[i] = a.cu[i];
+        __syncthreads();
+    }
+    const int32_t* __restrict__ cu = cu_in_smem ? s_cu : a.cu;
     const int lane = threadIdx.x & 31;
     const long long warps = (long long)gridDim.x * (kAppendThreads / 32);
     const uint4* __restrict__ kn = a.k_new;
@@ -48,8 +59,8 @@ __global__ void __launch_bounds__(kAppendThreads) kv_append_kernel(const AppendA
     uint4* __restrict__ kp = a.k_pool;
     uint4* __restrict__ vp = a.v_pool;
     for (long long t = (long long)blockIdx.x * (kAppendThreads / 32) + (threadIdx.x >> 5); t < a.T; t += warps) {
-        const int b = last_le(a.cu, a.B, t);
-        const long long pos = (long long)a.prefix[b] + (t - a.cu[b]);
+        const int b = last_le(cu, a.B, t);
+        const long long pos = (long long)a.prefix[b] + (t - cu[b]);
         const int page = a.page_table[(long long)b * a.max_pages + pos / a.ps];
         if (page < 0 || (long long)page >= a.num_pages) {
             if (lane == 0) atomicCAS(a.err, 0, RR_ERR_OOB);
