@@ -630,10 +630,13 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                 }
                 const long long src = (long long)(cu_b + t0 + t) * a.row16 + g * kPerTok + v;
                 const long long dst = (((long long)pid << ps_shift) + (pos & (a.ps - 1))) * a.row16 + g * kPerTok + v;
+                // streaming (evict-first) on both sides: nothing in this launch reads these lines again, and
+                // with default-policy stores the 2 x T x Hkv x D x 2 bytes pushed the units' shared K/V out of
+                // L2 (measured: 5 % of the step on c2, c4 and c5)
                 const uint4 kx = __ldcs(a.knew + src);
                 const uint4 vx = __ldcs(a.vnew + src);
-                a.kpool[dst] = kx;
-                a.vpool[dst] = vx;
+                __stcs(a.kpool + dst, kx);
+                __stcs(a.vpool + dst, vx);
             }
         }
     }
