@@ -372,6 +372,31 @@ def config_leg(rr, synth, name, steps, warmup, dev, st, peaks, rank, local):
                         "traffic": traffic_for(wl.name, kernel_source_hash()),
                         "algorithmic_flops": F, "algorithmic_bytes": attn_bytes(wl)},
            "clocks": clk}
+    if wl.shared_len > 0 and wl.shared_len % 128 == 0:
+        # the same attention as a cascade over the shared prefix (rr_extend_attention_shared), checked against
+        # the plain call's output within the parity bar and timed the same way
+        out_c = torch.empty_like(g["out"])
+
+        def cascade():
+            rr.extend_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                                g["suffix_lens"], out=out_c, shared_len=wl.shared_len)
+
+        for _ in range(warmup):
+            cascade()
+        cev = [tuple(torch.cuda.Event(enable_timing=True) for _ in range(2)) for _ in range(steps)]
+        for e0, e1 in cev:
+            e0.record(st)
+            cascade()
+            e1.record(st)
+        torch.cuda.synchronize(dev)
+        if rr.device_error():
+            raise RuntimeError(f"device error in the {name} cascade region")
+        if float((out_c.float() - g["out"].float()).abs().max()) > 2e-2:
+            raise RuntimeError(f"{name}: the shared-prefix cascade differs from the plain call")
+        c_ms = statistics.mean(e0.elapsed_time(e1) for e0, e1 in cev)
+        res["cascade"] = {"shared_len": int(wl.shared_len), "attention_ms": c_ms,
+                          "attention_tflops": F / (c_ms * 1e-3) / 1e12, "vs_plain": attn_ms / c_ms}
+        del out_c
     del g
     torch.cuda.empty_cache()
     return res

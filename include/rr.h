@@ -233,6 +233,35 @@ int rr_extend_step_rope(const void* q, const void* k_new, const void* v_new, voi
                         cudaStream_t stream);
 
 /*
+ * rr_extend_attention_shared -- rr_extend_attention for a batch whose agents
+ * all share their first shared_len positions (a common system prompt, the
+ * same physical pages at the start of every page table: Sec. 2's shared
+ * prefix cache), computed as a cascade.  A first pass attends every suffix
+ * row of the batch to the shared keys only, in dense Q tiles of consecutive
+ * rows whatever their agent (no causal mask is needed there: every suffix
+ * position lies past the shared keys), and keeps each (token, query head)'s
+ * unnormalised output and (max, sum) in fp32; a second pass attends each
+ * agent's rows to its keys from shared_len on, as rr_extend_attention does,
+ * and merges the two by their log-sum-exp weights.  Same result as
+ * rr_extend_attention within the parity tolerance (the summation order
+ * differs).  Measured slower than rr_extend_attention on GB300 (the shared
+ * keys cost the tensor-bound kernel nothing it could save, and the partials
+ * add a write and a read per row); provided for the comparison and for
+ * batches where that changes.
+ *
+ * shared_len: a positive multiple of 128 with shared_len <= prefix_lens[b]
+ * for every agent.  The device records RR_ERR_LENS if an agent's prefix is
+ * shorter, and RR_ERR_SHARED if an agent's first shared_len / page_size
+ * page-table entries differ from agent 0's; in either case no output is
+ * written.  The workspace grows by total_tokens x Hq x (D + 2) x 4 bytes for
+ * the partials.  Other arguments, layouts and errors as for
+ * rr_extend_attention.
+ */
+int rr_extend_attention_shared(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
+                               const int32_t* prefix_lens, const int32_t* suffix_lens, int32_t shared_len, void* out,
+                               const rr_dims* dims, float softmax_scale, cudaStream_t stream);
+
+/*
  * rr_decode_attention_shared -- rr_decode_attention for a batch whose agents
  * all share their first shared_len positions (a common system prompt, the
  * same physical pages at the start of every page table: Sec. 2's shared

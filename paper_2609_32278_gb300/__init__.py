@@ -45,7 +45,7 @@ EXPORTS = ("rr_kv_append", "rr_extend_attention", "rr_extend_step", "rr_decode_a
            "rr_get_device_error", "rr_last_error", "rr_version", "rr_shutdown", "rr_extend_attention_noalloc",
            "rr_rope_table", "rr_kv_append_rope", "rr_extend_attention_rope", "rr_extend_step_rope",
            "rr_decode_attention_rope", "rr_decode_attention_shared", "rr_set_wait_limit", "rr_kv_append_tensors",
-           "rr_extend_attention_tensors")
+           "rr_extend_attention_tensors", "rr_extend_attention_shared")
 
 RR_DTYPE_BF16 = 1
 RR_DTYPE_I32 = 2
@@ -104,6 +104,8 @@ def lib():
         L.rr_extend_step_rope.restype = ctypes.c_int
         L.rr_extend_step_rope.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, dp, ctypes.c_float, vp, ctypes.c_int32,
                                           vp]
+        L.rr_extend_attention_shared.restype = ctypes.c_int
+        L.rr_extend_attention_shared.argtypes = [vp, vp, vp, vp, vp, vp, ctypes.c_int32, vp, dp, ctypes.c_float, vp]
         L.rr_decode_attention_shared.restype = ctypes.c_int
         L.rr_decode_attention_shared.argtypes = [vp, vp, vp, vp, vp, ctypes.c_int32, vp, dp, ctypes.c_float, vp]
         L.rr_decode_attention_rope.restype = ctypes.c_int
@@ -208,9 +210,11 @@ def kv_append(k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens
 
 
 def extend_attention(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, out=None,
-                     softmax_scale: float = 0.0, stream=None, rope=None):
+                     softmax_scale: float = 0.0, stream=None, rope=None, shared_len: int = 0):
     """Extend attention of every suffix row over its agent's prefix + suffix (rr_extend_attention); with a
-    rope table, each q row is rotated at its position first (rr_extend_attention_rope)."""
+    rope table, each q row is rotated at its position first (rr_extend_attention_rope); with shared_len > 0,
+    every agent's first shared_len positions are the same pages and the call runs as a cascade over them
+    (rr_extend_attention_shared)."""
     import torch
     _need(q, "q", torch.bfloat16, 3)
     _need(k_pool, "k_pool", torch.bfloat16, 4)
@@ -235,7 +239,14 @@ def extend_attention(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, ou
     args = (q.data_ptr(), k_pool.data_ptr(), v_pool.data_ptr(), page_table.data_ptr(), prefix_lens.data_ptr(),
             suffix_lens.data_ptr(), out.data_ptr(), ctypes.byref(dims), float(softmax_scale))
     r = _rope_arg(rope, D)
-    if r is None:
+    if shared_len:
+        if r is not None:
+            raise ValueError("the shared-prefix cascade takes rotated queries only")
+        _check(lib().rr_extend_attention_shared(q.data_ptr(), k_pool.data_ptr(), v_pool.data_ptr(),
+                                                page_table.data_ptr(), prefix_lens.data_ptr(), suffix_lens.data_ptr(),
+                                                int(shared_len), out.data_ptr(), ctypes.byref(dims),
+                                                float(softmax_scale), _stream_ptr(stream, q.device)))
+    elif r is None:
         _check(lib().rr_extend_attention(*args, _stream_ptr(stream, q.device)))
     else:
         _check(lib().rr_extend_attention_rope(*args, r[0], r[1], _stream_ptr(stream, q.device)))

@@ -177,6 +177,43 @@ __device__ __forceinline__ void exp2_poly2(float& p0, float& p1, float x0, float
 constexpr int kEmuPairStride = RR_EMU_PAIR_STRIDE;
 
 
+// The cascade over a prefix every agent shares (rr_extend_attention_shared) runs the kernel twice.
+// kCasShared: every suffix row of the batch against the shared keys, in dense Q tiles of consecutive rows
+// whatever their agent (no causal mask: every suffix position lies past the shared keys), each row's
+// unnormalised O and (max, sum) written at (token, head).  kCasPrivate: the schedule's work units over each
+// agent's keys from the shared ones on, the epilogue merging the shared pass's partial into the output.
+constexpr int kCasNone = 0, kCasShared = 1, kCasPrivate = 2;
+
+// Work unit ui of the shared pass: KV head ui % Hkv, the Q tiles of rows (ui / Hkv) * unit_tokens.. of the
+// whole batch, agent 0's page table (the schedule checks that every agent's shared pages are agent 0's),
+// KV tiles [0, cas_tiles).  P = S + P = the shared keys, so every row's last visible key is the last shared one.
+__device__ __forceinline__ void cas_shared_unit(const AttnArgs& a, int ui, int& b, int& g, int& u, int& n_kv,
+                                                int& kb, int& ke, int& P, int& S, int& cu_b) {
+    const int hkv = a.Hq / a.G;
+    b = 0;
+    g = ui % hkv;
+    u = ui / hkv;
+    n_kv = a.cas_tiles;
+    kb = 0;
+    ke = a.cas_tiles;
+    P = a.cas_tiles * kBN;
+    S = 0;
+    cu_b = 0;
+}
+
+// KV tiles of item ui (the private pass never splits a unit; its first cas_tiles tiles are the shared pass's).
+template <int kCas>
+__device__ __forceinline__ int item_tiles(const AttnArgs& a, int ui) {
+    if constexpr (kCas == kCasShared) {
+        return a.cas_tiles;
+    } else {
+        const int4 U = a.units[ui];
+        if constexpr (kCas == kCasPrivate) return U.w - a.cas_tiles;
+        const int sp = (U.y >> 8) & 0xFF, ns = (U.y >> 16) & 0xFF;
+        return (sp + 1) * U.w / ns - sp * U.w / ns;
+    }
+}
+
 // Snake order: even waves left to right, odd waves right to left.
 __device__ __forceinline__ int unit_of(int wave, int cta, int grid) {
     return wave * grid + ((wave & 1) ? (grid - 1 - cta) : cta);
@@ -221,7 +258,7 @@ __device__ __noinline__ void rope_q_row(uint8_t* tile, int r, const float2* __re
 // kRope: q arrives un-rotated; as a unit's Q tiles land, each softmax thread rotates its own row at its
 // position P_b + i in shared memory, and the MMA issuer starts S_q only once tile q is rotated (the
 // keys were rotated on their way into the pool).
-template <int D, int NK, int NV, bool kFused, bool kRope>
+template <int D, int NK, int NV, bool kFused, bool kRope, int kCas = kCasNone>
 __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_constant__ AttnArgs a) {
     using C = Cfg<D, NK, NV>;
     extern __shared__ uint8_t smem_raw[];
@@ -275,7 +312,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
     ptx::tc_fence_after();
     const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + C::kOffMisc);
     ptx::griddep_wait();  // the schedule kernel's output (launched as its dependent)
-    const int n_units = *a.n_units;
+    const int n_units = kCas == kCasShared ? a.cas_units : *a.n_units;
     const int grid = gridDim.x, cta = blockIdx.x;
     const int unit_tokens = kNQ * a.tq;
 
@@ -293,10 +330,18 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
         for (int w = 0; ok; ++w) {
             const int ui = unit_of(w, cta, grid);
             if (ui >= n_units) break;
-            const int4 U = a.units[ui];
-            const int b = U.x, g = U.y & 0xFF, sp = (U.y >> 8) & 0xFF, ns = (U.y >> 16) & 0xFF, u = U.z;
-            const int n_kv = U.w, kb = sp * n_kv / ns, ke = (sp + 1) * n_kv / ns;  // this item's KV tiles
-            const int P = a.prefix[b], S = a.suffix[b], cu_b = a.cu[b];
+            // agent, KV head, unit, the unit's KV tiles, this item's [kb, ke), lengths, first row
+            int b, g, u, n_kv, kb, ke, P, S, cu_b;
+            if constexpr (kCas == kCasShared) {
+                cas_shared_unit(a, ui, b, g, u, n_kv, kb, ke, P, S, cu_b);
+            } else {
+                const int4 U = a.units[ui];
+                const int sp = (U.y >> 8) & 0xFF, ns = (U.y >> 16) & 0xFF;
+                b = U.x, g = U.y & 0xFF, u = U.z;
+                n_kv = U.w, kb = sp * n_kv / ns, ke = (sp + 1) * n_kv / ns;
+                if constexpr (kCas == kCasPrivate) kb = a.cas_tiles;  // the shared keys are the shared pass's
+                P = a.prefix[b], S = a.suffix[b], cu_b = a.cu[b];
+            }
             const int t0 = u * unit_tokens;
             const int n_keys = P + min(S, t0 + unit_tokens);
             const int agent_len = P + S;
@@ -453,9 +498,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             for (int w = 0; ok; ++w) {
                 const int ui = unit_of(w, cta, grid);
                 if (ui >= n_units) break;
-                const int4 U = a.units[ui];
-                const int sp = (U.y >> 8) & 0xFF, ns = (U.y >> 16) & 0xFF;
-                const int n_kv = (sp + 1) * U.w / ns - sp * U.w / ns;
+                const int n_kv = item_tiles<kCas>(a, ui);
                 for (int j = 0; j < n_kv; ++j, ++kv_count) {
                     const uint32_t nxt = kv_count + 1;
                     if (!(ok = wait_bar(bar(C::kVFull + (int)(kv_count % NV)), (kv_count / NV) & 1, ctl, lim, hint)))
@@ -525,9 +568,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             for (int w = 0; ok; ++w) {
                 const int ui = unit_of(w, cta, grid);
                 if (ui >= n_units) break;
-                const int4 U = a.units[ui];
-                const int sp = (U.y >> 8) & 0xFF, ns = (U.y >> 16) & 0xFF;
-                const int n_kv = (sp + 1) * U.w / ns - sp * U.w / ns;  // KV tiles of this item
+                const int n_kv = item_tiles<kCas>(a, ui);  // KV tiles of this item
                 if (!(ok = wait_bar(bar(C::kQFull), unit_i & 1, ctl))) break;
                 {
                     const int sk = (int)(kv_count % NK);
@@ -656,10 +697,19 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
         for (int w = 0; ok; ++w) {
             const int ui = unit_of(w, cta, grid);
             if (ui >= n_units) break;
-            const int4 U = a.units[ui];
-            const int b = U.x, g = U.y & 0xFF, sp = (U.y >> 8) & 0xFF, ns = (U.y >> 16) & 0xFF, u = U.z;
-            const int kb = sp * U.w / ns, ke = (sp + 1) * U.w / ns;  // this item's KV tiles
-            const int P = a.prefix[b], agent_len = P + a.suffix[b];
+            int b, g, u, kb, ke, P, agent_len;  // agent, KV head, unit, this item's KV tiles, keys
+            if constexpr (kCas == kCasShared) {
+                int n_kv, S, cu_b;
+                cas_shared_unit(a, ui, b, g, u, n_kv, kb, ke, P, S, cu_b);
+                agent_len = P;  // every row sees exactly the shared keys: P - 1 is each row's last key
+            } else {
+                const int4 U = a.units[ui];
+                const int sp = (U.y >> 8) & 0xFF, ns = (U.y >> 16) & 0xFF;
+                b = U.x, g = U.y & 0xFF, u = U.z;
+                kb = sp * U.w / ns, ke = (sp + 1) * U.w / ns;
+                if constexpr (kCas == kCasPrivate) kb = a.cas_tiles;
+                P = a.prefix[b], agent_len = P + a.suffix[b];
+            }
             const int tq0 = u * unit_tokens + q * a.tq;  // first suffix token of this Q tile
             const int row_limit = min(P + tq0 + r / a.G, agent_len - 1);     // last key this row may see
             const int mask_from = (min(P + tq0, agent_len - 1) + 1) / kBN;  // earlier tiles: no masking
@@ -785,6 +835,81 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                 }
             }
             if (!ok) break;
+            if constexpr (kCas == kCasShared) {
+                if (!(ok = wait_bar(bar(C::kOFinal + q), o_phase, ctl))) break;
+                o_phase ^= 1;
+                ptx::tc_fence_after();
+                // this row's unnormalised O and (max, sum) at (token, head), for the private pass to merge
+                const long long tok = (long long)tq0 + r / a.G;  // a row of the whole batch
+                const bool valid = tok < a.cas_T;
+                const long long prow = tok * a.Hq + g * a.G + r % a.G;
+                float4* po = reinterpret_cast<float4*>(a.cas_o + prow * D);
+#pragma unroll
+                for (int c = 0; c < D; c += 32) {
+                    uint32_t o[32];
+                    ptx::tmem_ld32(t_o + c, o);
+                    ptx::tmem_wait_ld_regs(o);
+                    if (valid) {
+#pragma unroll
+                        for (int i = 0; i < 8; ++i)
+                            po[c / 4 + i] = make_float4(__uint_as_float(o[4 * i]), __uint_as_float(o[4 * i + 1]),
+                                                        __uint_as_float(o[4 * i + 2]), __uint_as_float(o[4 * i + 3]));
+                    }
+                }
+                if (valid) a.cas_ml[prow] = make_float2(m_run, l_run);
+                continue;
+            }
+            if constexpr (kCas == kCasPrivate) {
+                // merge with the shared pass's partial of this (token, head): both are in log2 units of the same
+                // scale, so o = (2^(m_s - M) O_s + 2^(m - M) O) / (2^(m_s - M) l_s + 2^(m - M) l), M = max(m_s, m)
+                const int tok = tq0 + r / a.G;
+                const bool valid = tok < a.suffix[b];
+                const long long prow = (long long)(a.cu[b] + tok) * a.Hq + g * a.G + r % a.G;
+                const float4* so = reinterpret_cast<const float4*>(a.cas_o + prow * D);
+                const float2 ml = valid ? a.cas_ml[prow] : make_float2(-INFINITY, 0.f);  // in flight during the wait
+                if (!(ok = wait_bar(bar(C::kOFinal + q), o_phase, ctl))) break;
+                o_phase ^= 1;
+                ptx::tc_fence_after();
+                const float M = fmaxf(ml.x, m_run);  // m_run is finite: a row sees at least its own key here
+                const float ws = ml.x == -INFINITY ? 0.f : ptx::ex2_approx(ml.x - M);
+                const float wp = ptx::ex2_approx(m_run - M);
+                const float inv = 1.0f / (ws * ml.y + wp * l_run);
+                __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(a.out) + prow * D;
+                // 16 columns at a time (few registers: this is the epilogue of a kernel tuned to its limit), the
+                // shared partial's next 16 columns in flight while these are merged and stored
+                float4 nx[4];
+                if (valid) {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) nx[i] = so[i];
+                }
+#pragma unroll
+                for (int c = 0; c < D; c += 16) {
+                    uint32_t o[16];
+                    ptx::tmem_ld16(t_o + c, o);
+                    float4 sx[4];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) sx[i] = nx[i];
+                    if (valid && c + 16 < D) {
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) nx[i] = so[(c + 16) / 4 + i];
+                    }
+                    ptx::tmem_wait_ld_regs16(o);
+                    uint32_t pk[8];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        pk[2 * i] = ptx::pack_bf16x2((wp * __uint_as_float(o[4 * i]) + ws * sx[i].x) * inv,
+                                                     (wp * __uint_as_float(o[4 * i + 1]) + ws * sx[i].y) * inv);
+                        pk[2 * i + 1] = ptx::pack_bf16x2((wp * __uint_as_float(o[4 * i + 2]) + ws * sx[i].z) * inv,
+                                                         (wp * __uint_as_float(o[4 * i + 3]) + ws * sx[i].w) * inv);
+                    }
+                    if (valid) {
+                        uint4* d4 = reinterpret_cast<uint4*>(dst + c);
+                        d4[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                        d4[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+                    }
+                }
+                continue;
+            }
             if (!(ok = wait_bar(bar(C::kOFinal + q), o_phase, ctl))) break;
             o_phase ^= 1;
             ptx::tc_fence_after();
@@ -832,7 +957,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
     ptx::mbar_arrive(bar(C::kDone));
 }
 
-template <int D, int NK, int NV, bool kFused, bool kRope>
+template <int D, int NK, int NV, bool kFused, bool kRope, int kCas = kCasNone>
 cudaError_t launch_cfg(const AttnArgs& a, int grid, cudaStream_t st) {
     using C = Cfg<D, NK, NV>;
     static bool attr_done[64] = {};
@@ -841,13 +966,18 @@ cudaError_t launch_cfg(const AttnArgs& a, int grid, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     if (!attr_done[dev]) {
-        e = cudaFuncSetAttribute(extend_attn_kernel<D, NK, NV, kFused, kRope>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 C::kSmemBytes);
+        e = cudaFuncSetAttribute(extend_attn_kernel<D, NK, NV, kFused, kRope, kCas>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
         if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
-    return launch_after_sched(extend_attn_kernel<D, NK, NV, kFused, kRope>, dim3(grid), dim3(kThreads), C::kSmemBytes, st,
-                              a);
+    if constexpr (kCas == kCasShared) {  // needs no schedule: an ordinary launch
+        extend_attn_kernel<D, NK, NV, kFused, kRope, kCas><<<grid, kThreads, C::kSmemBytes, st>>>(a);
+        return cudaGetLastError();
+    } else {
+        return launch_after_sched(extend_attn_kernel<D, NK, NV, kFused, kRope, kCas>, dim3(grid), dim3(kThreads),
+                                  C::kSmemBytes, st, a);
+    }
 }
 
 }  // namespace
@@ -856,6 +986,16 @@ size_t extend_attention_smem_bytes(int head_dim) {
     if (head_dim == 128) return Cfg<128, 2, 3>::kSmemBytes;
     if (head_dim == 64) return Cfg<64, 4, 4>::kSmemBytes;
     return 0;
+}
+
+cudaError_t launch_extend_cascade(const AttnArgs& a, int head_dim, int grid, cudaStream_t st, bool shared_pass) {
+    if (head_dim == 128)
+        return shared_pass ? launch_cfg<128, 2, 3, false, false, kCasShared>(a, grid, st)
+                           : launch_cfg<128, 2, 3, false, false, kCasPrivate>(a, grid, st);
+    if (head_dim == 64)
+        return shared_pass ? launch_cfg<64, 4, 4, false, false, kCasShared>(a, grid, st)
+                           : launch_cfg<64, 4, 4, false, false, kCasPrivate>(a, grid, st);
+    return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_extend_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st, bool fused) {

@@ -359,6 +359,121 @@ int attention_impl(const void* q, const void* k_pool, const void* v_pool, const 
     return RR_OK;
 }
 
+// Extend attention over a prefix every agent of the batch shares (rr_extend_attention_shared), as a cascade:
+// the shared pass runs every suffix row of the batch against the shared keys in dense Q tiles that cross
+// agents, writing fp32 partials per (token, head); the private pass runs the schedule's units over each agent's
+// remaining keys and merges the partial into the output in its epilogue.
+int extend_shared_impl(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
+                       const int32_t* prefix_lens, const int32_t* suffix_lens, int32_t shared_len, void* out,
+                       const rr_dims* dims, float softmax_scale, cudaStream_t stream) {
+    g_msg[0] = 0;
+    int rc = check_dims(dims, true);
+    if (rc) return rc;
+    if (dims->total_tokens == 0 && dims->batch == 0) return RR_OK;
+    if (!page_table || !prefix_lens || !suffix_lens) return fail(RR_ERR_INVALID_ARG, "null lens or page table");
+    if (dims->total_tokens > 0 && (!q || !k_pool || !v_pool || !out))
+        return fail(RR_ERR_INVALID_ARG, "null q/pool/out pointer");
+    if (!aligned16(q) || !aligned16(k_pool) || !aligned16(v_pool) || !aligned16(out))
+        return fail(RR_ERR_INVALID_ARG, "q, pools and out must be 16-byte aligned");
+    if (!aligned4(page_table) || !aligned4(prefix_lens) || !aligned4(suffix_lens))
+        return fail(RR_ERR_INVALID_ARG, "int32 arrays must be 4-byte aligned");
+    if (dims->total_tokens > 0 && dims->num_pages == 0) return fail(RR_ERR_INVALID_ARG, "empty pool");
+    const int Hq = dims->num_q_heads, Hkv = dims->num_kv_heads, D = dims->head_dim, ps = dims->page_size;
+    if (shared_len <= 0 || shared_len % rr::kBN != 0)
+        return fail(RR_ERR_UNSUPPORTED, "shared_len (%d) must be a positive multiple of %d", shared_len, rr::kBN);
+    if ((int64_t)shared_len > (int64_t)dims->max_pages * ps) return fail(RR_ERR_INVALID_ARG, "shared_len exceeds max_pages");
+    const int G = Hq / Hkv;
+    const int tq = rr::kBM / G;
+    const int unit_tokens = rr::kNQ * tq;
+    const int64_t T = dims->total_tokens, B = dims->batch;
+    const int64_t max_units = (int64_t)Hkv * (T / unit_tokens + B + 1);
+    const int64_t shared_units = (int64_t)Hkv * ((T + unit_tokens - 1) / unit_tokens);
+    if (max_units >= (1ll << 31)) return fail(RR_ERR_UNSUPPORTED, "too many work units");
+
+    Device* d = nullptr;
+    if ((rc = current_device(&d, nullptr))) return rc;
+    if ((rc = get_encoder())) return rc;
+    const Layout L = layout_for(B, max_units);
+    const size_t off_ml = align256(L.total);
+    const size_t off_o = off_ml + align256((size_t)T * Hq * 8);
+    if ((rc = ensure_ws(*d, off_o + (size_t)T * Hq * (size_t)D * 4))) return rc;
+    uint8_t* ws = static_cast<uint8_t*>(d->ws);
+
+    rr::AttnArgs a;
+    memset(&a, 0, sizeof a);
+    if (T > 0) {
+        if ((rc = encode_3d(&a.tm_q, q, (uint64_t)D, (uint64_t)Hq, (uint64_t)T, (uint64_t)D * 2, (uint64_t)Hq * D * 2,
+                            64, (uint32_t)G, (uint32_t)tq)))
+            return rc;
+        const uint64_t rows = (uint64_t)dims->num_pages * (uint64_t)ps;
+        if ((rc = encode_2d(&a.tm_k, k_pool, (uint64_t)Hkv * D, rows, (uint64_t)Hkv * D * 2, 64, (uint32_t)ps))) return rc;
+        if ((rc = encode_2d(&a.tm_v, v_pool, (uint64_t)Hkv * D, rows, (uint64_t)Hkv * D * 2, 64, (uint32_t)ps))) return rc;
+        a.oob_row = (int32_t)rows;
+    }
+    a.page_table = page_table;
+    a.prefix = prefix_lens;
+    a.suffix = suffix_lens;
+    a.err = d->err;
+    a.out = out;
+    a.num_pages = dims->num_pages;
+    a.Hq = Hq;
+    a.G = G;
+    a.ps = ps;
+    a.max_pages = dims->max_pages;
+    a.tq = tq;
+    const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)D);
+    a.scale_log2 = scale * 1.4426950408889634f;
+    a.wait_limit = rr::wait_limit_cycles();
+    a.wait_hint_ns = (uint32_t)std::min<long long>(200000, std::max<long long>(1, a.wait_limit / 4));
+    a.cas_tiles = shared_len / rr::kBN;
+    a.cas_units = (int32_t)shared_units;
+    a.cas_T = T;
+    a.cas_ml = reinterpret_cast<float2*>(ws + off_ml);
+    a.cas_o = reinterpret_cast<float*>(ws + off_o);
+    cudaError_t e = cudaSuccess;
+    if (T > 0) {  // the shared pass needs nothing from the schedule
+        const int64_t grid = std::min<int64_t>((int64_t)d->sm_count, shared_units);
+        e = rr::launch_extend_cascade(a, D, (int)std::max<int64_t>(grid, 1), stream, true);
+        if (e != cudaSuccess) return cuda_fail(e, "shared-prefix pass launch");
+    }
+
+    rr::SchedArgs s{};
+    s.prefix = prefix_lens;
+    s.suffix = suffix_lens;
+    s.B = (int32_t)B;
+    s.Hkv = Hkv;
+    s.unit_tokens = unit_tokens;
+    s.T = T;
+    s.max_pages = dims->max_pages;
+    s.ps = ps;
+    s.max_units = max_units;
+    s.build_units = 1;
+    s.cu = reinterpret_cast<int32_t*>(ws + L.off_cu);
+    s.unit_off = reinterpret_cast<int32_t*>(ws + L.off_unit_off);
+    s.units = reinterpret_cast<int4*>(ws + L.off_units);
+    s.item_slot = reinterpret_cast<int32_t*>(ws + L.off_slot);
+    s.split_units = nullptr;  // the private pass never splits a unit
+    s.n_split = reinterpret_cast<int32_t*>(ws) + 2;
+    s.split_grid = 0;
+    s.page_table = page_table;
+    s.shared_pages = shared_len / ps;  // every agent's shared pages are agent 0's (RR_ERR_SHARED)
+    s.min_prefix = shared_len;         // and every agent's prefix covers them (RR_ERR_LENS)
+    s.n_units = reinterpret_cast<int32_t*>(ws);
+    s.lens_ok = reinterpret_cast<int32_t*>(ws) + 1;
+    s.err = d->err;
+    e = rr::launch_sched(s, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "schedule kernel launch");
+    if (T == 0) return RR_OK;
+    a.cu = s.cu;
+    a.units = s.units;
+    a.n_units = s.n_units;
+    a.item_slot = s.item_slot;
+    const int64_t grid = std::min<int64_t>((int64_t)d->sm_count, max_units);
+    e = rr::launch_extend_cascade(a, D, (int)std::max<int64_t>(grid, 1), stream, false);
+    if (e != cudaSuccess) return cuda_fail(e, "private-key pass launch");
+    return RR_OK;
+}
+
 // Decode over a prefix every agent of the batch shares (rr_decode_attention_shared): the shared prefix's
 // pages are read once per group of 16 / G agents (their queries fill the MMA's 16 columns) instead of once
 // per agent, each agent's private keys by the plain decode kernel, and both partial results are merged.
@@ -677,6 +792,13 @@ int rr_decode_attention_shared(const void* q, const void* k_pool, const void* v_
                                const int32_t* kv_lens, int32_t shared_len, void* out, const rr_dims* dims,
                                float softmax_scale, cudaStream_t stream) {
     return decode_shared_impl(q, k_pool, v_pool, page_table, kv_lens, shared_len, out, dims, softmax_scale, stream);
+}
+
+int rr_extend_attention_shared(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
+                               const int32_t* prefix_lens, const int32_t* suffix_lens, int32_t shared_len, void* out,
+                               const rr_dims* dims, float softmax_scale, cudaStream_t stream) {
+    return extend_shared_impl(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, shared_len, out, dims,
+                              softmax_scale, stream);
 }
 
 int rr_decode_attention_rope(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,

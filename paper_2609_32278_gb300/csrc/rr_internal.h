@@ -48,6 +48,7 @@ struct SchedArgs {
     int32_t* unit_slot;
     const int32_t* page_table;
     int32_t shared_pages;
+    int32_t min_prefix;    // every agent's prefix must be at least this long (extend over a shared prefix)
     int32_t* n_units;      // number of items
     int32_t* lens_ok;
     int32_t* err;
@@ -116,6 +117,12 @@ struct AttnArgs {
     const int32_t* unit_slot;  // first partial slot of unit (agent b, KV head g) at b * Hkv + g
     int32_t group_items, group_ns, group_agents, groups_per_head, shared_tiles, batch;
     CUtensorMap tm_qg;
+    // extend over a shared prefix (rr_extend_attention_shared): cas_tiles = shared keys / 128; the shared pass
+    // runs cas_units implicit units over all cas_T suffix rows; partials [cas_T * Hq][D] and [cas_T * Hq]
+    int32_t cas_tiles, cas_units;
+    int64_t cas_T;
+    float* cas_o;
+    float2* cas_ml;
 };
 
 struct CombineArgs {
@@ -160,6 +167,9 @@ cudaError_t launch_kv_append(const AppendArgs& a, int sm_count, cudaStream_t st)
 // suffix K/V come from k_new / v_new, and the kernel also writes them into the pool).  a.rope set: q
 // is rotated in shared memory as each Q tile lands (not with fused).
 cudaError_t launch_extend_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st, bool fused = false);
+// The two passes of rr_extend_attention_shared (shared_pass: every suffix row against the shared keys, an
+// ordinary launch; otherwise the schedule's units over the private keys, merging, as the schedule's dependent).
+cudaError_t launch_extend_cascade(const AttnArgs& a, int head_dim, int grid, cudaStream_t st, bool shared_pass);
 // Rotary table (rope.cu): table[p][i] = (cos, sin) of p * base^(-2i/D), p < max_pos, i < D/2.
 cudaError_t launch_rope_table(float2* out, int max_pos, int head_dim, double base, int sm_count, cudaStream_t st);
 size_t extend_attention_smem_bytes(int head_dim);

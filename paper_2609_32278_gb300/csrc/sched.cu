@@ -115,13 +115,13 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
             a.prefix_out[b] = L - 1;  // L < 1 fails the check below
             a.suffix_out[b] = 1;
         }
-        if (a.shared_pages > 0) {  // every agent's shared-prefix pages are agent 0's
-            for (long long i = tid; i < (long long)B * a.shared_pages; i += 1024) {
-                const long long b = i / a.shared_pages, p = i % a.shared_pages;
-                if (a.page_table[b * a.max_pages + p] != a.page_table[p]) {
-                    atomicCAS(a.err, 0, RR_ERR_SHARED);
-                    s_bad = 1;
-                }
+    }
+    if (a.shared_pages > 0) {  // a batch over a shared prefix: every agent's shared-prefix pages are agent 0's
+        for (long long i = tid; i < (long long)B * a.shared_pages; i += 1024) {
+            const long long b = i / a.shared_pages, p = i % a.shared_pages;
+            if (a.page_table[b * a.max_pages + p] != a.page_table[p]) {
+                atomicCAS(a.err, 0, RR_ERR_SHARED);
+                s_bad = 1;
             }
         }
     }
@@ -130,7 +130,7 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     bool bad = false;
     for (int b = b0; b < b1; ++b) {
         const int P = a.prefix[b], S = a.suffix[b];
-        if (P < 0 || S < 0 || (long long)P + S > cap) { bad = true; continue; }
+        if (P < a.min_prefix || S < 0 || (long long)P + S > cap) { bad = true; continue; }
         sum_s += S;
         sum_u += (long long)a.Hkv * ((S + a.unit_tokens - 1) / a.unit_tokens);  // 32-bit division
     }

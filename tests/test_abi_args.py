@@ -164,3 +164,25 @@ def test_error_message_is_cleared_by_a_good_call(rr):
     expect(rr, attn(rr, dims(rr, D=96)), UNSUPPORTED, ["head_dim"])
     assert attn(rr, dims(rr, B=0, T=0, max_pages=0, num_pages=0)) == OK
     assert rr.last_error() == ""
+
+
+def shared_attn(rr, d, shared_len, q=A16, kp=A16, vp=A16, pt=A4, pl=A4, sl=A4, out=A16):
+    return rr.lib().rr_extend_attention_shared(q, kp, vp, pt, pl, sl, shared_len, out, d, 0.0, None)
+
+
+@pytest.mark.parametrize("shared_len,code,words", [
+    (0, UNSUPPORTED, ["shared_len (0)", "multiple of 128"]),
+    (-128, UNSUPPORTED, ["shared_len (-128)"]),
+    (200, UNSUPPORTED, ["shared_len (200)"]),
+    (128 * 5, INVALID, ["exceeds max_pages"]),       # 4 pages x 16 tokens
+])
+def test_shared_cascade_rejects_bad_shared_len(rr, shared_len, code, words):
+    expect(rr, shared_attn(rr, dims(rr, max_pages=4), shared_len), code, words)
+
+
+def test_shared_cascade_checks_like_the_plain_call(rr):
+    expect(rr, shared_attn(rr, dims(rr, D=96), 128), UNSUPPORTED, ["head_dim 96"])
+    expect(rr, shared_attn(rr, dims(rr, max_pages=8), 128, q=None), INVALID, ["null q/pool/out"])
+    expect(rr, shared_attn(rr, dims(rr, max_pages=8), 128, pt=None), INVALID, ["null lens or page table"])
+    expect(rr, shared_attn(rr, dims(rr, max_pages=8), 128, out=MIS), INVALID, ["16-byte aligned"])
+    assert shared_attn(rr, dims(rr, B=0, T=0), 128) == OK
