@@ -677,7 +677,7 @@ def run_ours(args, world, rank, local):
     value = world * F / (ms_step * 1e-3) / 1e12
     tok_s = world * wl.T / (ms_step * 1e-3)
 
-    # ---- the same step as one launch (rr_extend_step: append fused into the attention kernel)
+    # ---- the same step as one launch (rr_extend_step: the kernel appends, crosses a grid barrier, attends)
     fused = None
     if not args.no_fused:
         fev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
@@ -797,6 +797,25 @@ def run_ours(args, world, rank, local):
                 "attention_ms": r_att, "attention_tflops": F / (r_att * 1e-3) / 1e12, "kv_append_ms": r_app,
                 "kv_append_gbs": append_bytes(wl) / (r_app * 1e-3) / 1e9, "vs_plain_step": ms_step / r_ms,
                 "base": 500000.0}
+        if not args.no_fused:  # the same rotated step as one launch (rr_extend_step_rope)
+            def rope_one():
+                rr.extend_step(g["q"], g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"],
+                               g["prefix_lens"], g["suffix_lens"], out=out_r, rope=table)
+
+            for _ in range(args.warmup):
+                rope_one()
+            torch.cuda.synchronize(dev)
+            oev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+            for e0, e1 in oev:
+                e0.record(st)
+                rope_one()
+                e1.record(st)
+            torch.cuda.synchronize(dev)
+            if rr.device_error():
+                raise RuntimeError("device error in the one-launch rotary-step region")
+            o_ms = max_over_ranks(statistics.mean(e0.elapsed_time(e1) for e0, e1 in oev), world, dev)
+            rope.update({"one_launch_ms": o_ms, "one_launch_value": world * F / (o_ms * 1e-3) / 1e12,
+                         "one_launch_vs_two_calls": r_ms / o_ms})
         # restore the un-rotated suffix keys for the legs that follow
         rr.kv_append(g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
                      g["suffix_lens"])

@@ -116,19 +116,21 @@ int rr_extend_attention(const void* q, const void* k_pool, const void* v_pool, c
  * rr_extend_step -- the whole extend step of Sec. 2 in one attention launch:
  * the same results as rr_kv_append followed by rr_extend_attention on the
  * same stream (the pools receive the suffix K/V bit for bit, and `out` is
- * bit-identical), without the separate pass over k_new / v_new.
+ * bit-identical), with two kernels launched instead of four.
  *
- * The attention kernel reads every suffix position's K/V straight from
- * k_new / v_new [T][Hkv][D] (cached positions from the pool through
- * page_table, as before), and each work unit also writes its own suffix rows
- * into the pool slots page_table assigns to them, for later calls.  Arguments,
- * layouts, preconditions and errors are those of the two calls it replaces;
- * k_pool / v_pool are written, so they are non-const here.
+ * The kernel first writes every suffix row of k_new / v_new [T][Hkv][D] into
+ * the pool slots page_table assigns to it, with all its threads; then every
+ * CTA waits at a grid-wide barrier (the kernel is launched cooperatively, one
+ * CTA per SM, so all of them are resident); then it runs the attention over
+ * the pool.  The barrier's wait is bounded like the pipeline's waits
+ * (rr_set_wait_limit): if it runs out, RR_ERR_TIMEOUT is recorded and the
+ * output is undefined.  Arguments, layouts, preconditions and errors are those
+ * of the two calls it replaces; k_pool / v_pool are written, so they are
+ * non-const here.
  *
- * Performance: it launches two kernels where the two calls launch four, which
- * makes it faster for a small extend (one agent, a few thousand keys: ~1.1x
- * measured on GB300), and slower for large batches (~0.9x), where the
- * separate append pass it saves is well under 1 % of the step.
+ * Performance (GB300): 1.01-1.03x the two calls on the long-context batches,
+ * and up to ~1.09x on a single small extend (one agent, a few thousand keys),
+ * where the saved launches matter most.
  */
 int rr_extend_step(const void* q, const void* k_new, const void* v_new, void* k_pool, void* v_pool,
                    const int32_t* page_table, const int32_t* prefix_lens, const int32_t* suffix_lens, void* out,
@@ -221,11 +223,13 @@ int rr_extend_attention_rope(const void* q, const void* k_pool, const void* v_po
                              cudaStream_t stream);
 
 /*
- * rr_extend_step_rope -- the extend step with rotary embedding:
- * rr_kv_append_rope followed by rr_extend_attention_rope on `stream` (two
- * launches after their schedules; the one-launch rr_extend_step reads the
- * suffix keys straight from k_new, which would need rotating in shared memory
- * on every tile, so it takes rotated rows only).
+ * rr_extend_step_rope -- the extend step with rotary embedding in one
+ * launch: the same results as rr_kv_append_rope followed by
+ * rr_extend_attention_rope on `stream` (pools and `out` bit-identical).  The
+ * kernel's first phase rotates each K row at its position P_b + j as it
+ * writes the pool (the same arithmetic as rr_kv_append_rope); after the grid
+ * barrier the attention rotates q as each Q tile lands.  Other arguments,
+ * preconditions and errors as for rr_extend_step and rr_kv_append_rope.
  */
 int rr_extend_step_rope(const void* q, const void* k_new, const void* v_new, void* k_pool, void* v_pool,
                         const int32_t* page_table, const int32_t* prefix_lens, const int32_t* suffix_lens, void* out,

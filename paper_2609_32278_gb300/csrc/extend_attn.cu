@@ -81,7 +81,6 @@ static_assert((2 * kRegsSoftmax + kRegsControl) * 32 <= 16384, "register split e
 constexpr int kWarpProducer = 8;
 constexpr int kWarpMMA = 9;
 constexpr int kWarpStage = 10;
-constexpr int kWarpAppend = 11;  // fused extend step: writes each unit's suffix K/V into the pool
 constexpr long long kWaitLimitCycles = 1ll << 33;  // ~4 s at 2 GHz
 
 template <int D, int NK, int NV>
@@ -99,8 +98,7 @@ struct Cfg {
     static constexpr int kKFull = 2, kKEmpty = 2 + NK, kVFull = 2 + 2 * NK, kVEmpty = 2 + 2 * NK + NV;
     static constexpr int kSFull = 2 + 2 * NK + 2 * NV, kPFull = kSFull + kNQ, kOFinal = kPFull + kNQ;
     static constexpr int kVTmp = kOFinal + kNQ, kDrain = kVTmp + 1, kDone = kDrain + 1;
-    static constexpr int kKTmp = kDone + 1;  // fused step: a K tile that needs fixing up before release
-    static constexpr int kQRot = kKTmp + 1;  // rotary q: Q tile q rotated in shared memory (kNQ barriers)
+    static constexpr int kQRot = kDone + 1;  // rotary q: Q tile q rotated in shared memory (kNQ barriers)
     static constexpr int kNumBars = kQRot + kNQ;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // u32 TMEM base, i32 abort flag
     static constexpr int kSmemBytes = kOffMisc + 16 + 1024;  // + slack to align the base to 1 KiB
@@ -252,9 +250,123 @@ __device__ __noinline__ void rope_q_row(uint8_t* tile, int r, const float2* __re
     }
 }
 
-// kFused: the one-launch extend step.  Suffix positions' K/V are read from k_new / v_new (the caller's
-// rows, not the pool), and warp 11 writes each work unit's own suffix rows into the pool, so no unit
-// waits for another CTA's pool writes; the attention result is bit-identical to append-then-attend.
+// Phase 1 of the one-launch extend step: every suffix row of every KV head goes to its pool slot, K
+// rotated at the row's position P_b + i when a rotary table is given, the same bytes rr_kv_append /
+// rr_kv_append_rope write; then the grid waits until all of it is written, so that phase 2, the plain
+// attention pipeline over the pool, finds each suffix key where a separate append would have put it.
+// The work is handed out in tasks of 8 tokens of one unit's KV head over every warp of the grid (only
+// units with split index 0: each (token, KV head) belongs to exactly one), with all of a lane's loads
+// in flight before its stores.  Streaming (evict-first) loads and stores: this launch reads no k_new /
+// v_new line again, and default-policy pool stores would push prefix K/V out of L2.
+// The barrier needs every CTA resident at once (a cooperative launch, one CTA per SM); its spin is
+// bounded by a.wait_limit, after which it reports RR_ERR_TIMEOUT and returns 0: the CTA then runs no
+// unit of phase 2 (it still sets up and tears down its pipeline, so that every role ends as usual).
+// Code generation note: the pipeline after this phase is sensitive to how the kernel gets past it.
+// Leaving the kernel here on a failed barrier (before the mbarrier initialisation and the tensor-memory
+// allocation), or ignoring the outcome, each made the whole step 7-8 % slower on the c2, c4 and c5
+// batches than this form, in which the outcome only zeroes the unit count.
+template <int D, bool kRope>
+__device__ __forceinline__ int fused_append(const AttnArgs& a, int n_units, int unit_tokens) {
+    constexpr int kPerTok = D / 8;  // 16-byte vectors of one head's row
+    constexpr int kTask = 8;        // tokens per warp task (unit_tokens = 256 / G is a multiple of 16)
+    const int lane = threadIdx.x & 31;
+    const long long n_warps = (long long)gridDim.x * (kThreads / 32);
+    const int tasks_per_unit = unit_tokens / kTask;
+    const int ps_shift = __ffs(a.ps) - 1;  // page sizes are powers of two
+    for (long long c = (long long)blockIdx.x * (kThreads / 32) + (threadIdx.x >> 5); c < (long long)n_units * tasks_per_unit;
+         c += n_warps) {
+        const int ui = (int)(c / tasks_per_unit);
+        const int4 U = a.units[ui];
+        if (((U.y >> 8) & 0xFF) != 0) continue;  // a later piece of a split unit
+        const int b = U.x, g = U.y & 0xFF;
+        const int P = a.prefix[b], S = a.suffix[b];
+        const int t0 = U.z * unit_tokens + (int)(c - (long long)ui * tasks_per_unit) * kTask;
+        const int n = min(kTask, S - t0);
+        if (n <= 0) continue;
+        const int32_t* pt = a.page_table + (long long)b * a.max_pages;
+        const long long src0 = (long long)(a.cu[b] + t0) * a.row16 + g * kPerTok;
+        // the pool row of token t of the task (-1: not written, the error reported)
+        auto dst_row = [&](int t) -> long long {
+            if (t >= n) return -1;
+            const int pos = P + t0 + t;
+            if (kRope && pos >= a.rope_max_pos) {
+                atomicCAS(a.err, 0, RR_ERR_LENS);
+                return -1;
+            }
+            const int pid = pt[pos >> ps_shift];
+            if (pid < 0 || (long long)pid >= a.num_pages) {
+                atomicCAS(a.err, 0, RR_ERR_OOB);
+                return -1;
+            }
+            return (((long long)pid << ps_shift) + (pos & (a.ps - 1))) * a.row16 + g * kPerTok;
+        };
+        {  // V, and K without a rotary table: one vector per lane and pass
+            constexpr int kTokPerPass = 32 / kPerTok, kPasses = kTask / kTokPerPass;
+            const int sub = lane / kPerTok, v = lane % kPerTok;
+            long long dst[kPasses];
+            uint4 kx[kPasses], vx[kPasses];
+#pragma unroll
+            for (int p = 0; p < kPasses; ++p) {
+                const int t = p * kTokPerPass + sub;
+                dst[p] = dst_row(t);
+                if (dst[p] >= 0) {
+                    const long long src = src0 + (long long)t * a.row16 + v;
+                    if (!kRope) kx[p] = __ldcs(a.knew + src);
+                    vx[p] = __ldcs(a.vnew + src);
+                }
+            }
+#pragma unroll
+            for (int p = 0; p < kPasses; ++p) {
+                if (dst[p] < 0) continue;
+                if (!kRope) __stcs(a.kpool + dst[p] + v, kx[p]);
+                __stcs(a.vpool + dst[p] + v, vx[p]);
+            }
+        }
+        if constexpr (kRope) {  // K: the two vectors of one rotation pair (elements 8u.. and 8u + D/2..) per lane
+            constexpr int kHalf = kPerTok / 2, kTokPerPass = 32 / kHalf, kPasses = kTask / kTokPerPass;
+            const int sub = lane / kHalf, u = lane % kHalf;
+#pragma unroll
+            for (int p = 0; p < kPasses; ++p) {
+                const int t = p * kTokPerPass + sub;
+                const long long dst = dst_row(t);
+                if (dst < 0) continue;
+                const long long src = src0 + (long long)t * a.row16;
+                uint4 k0 = __ldcs(a.knew + src + u), k1 = __ldcs(a.knew + src + u + kHalf);
+                float4 cs[4];
+                rope_load8(cs, a.rope + (long long)(P + t0 + t) * (D / 2) + 8 * u);
+                rope_rotate8(k0, k1, cs);
+                __stcs(a.kpool + dst + u, k0);
+                __stcs(a.kpool + dst + u + kHalf, k1);
+            }
+        }
+    }
+    // grid barrier: every CTA's pool stores, then its arrival; the attention reads the rows through TMA
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+    __syncthreads();
+    int ok = 1;
+    if (threadIdx.x == 0) {
+        __threadfence();
+        atomicAdd(a.grid_sync, 1);
+        const long long t_start = clock64();
+        for (;;) {
+            int arrived;
+            asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(arrived) : "l"(a.grid_sync) : "memory");
+            if (arrived >= (int)gridDim.x) break;
+            if (clock64() - t_start > a.wait_limit) {
+                atomicCAS(a.err, 0, RR_ERR_TIMEOUT);
+                ok = 0;
+                break;
+            }
+            __nanosleep(100);
+        }
+    }
+    ok = __syncthreads_and(ok);
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+    return ok;
+}
+
+// kFused: the one-launch extend step, fused_append above and then the attention over the pool; the
+// result is bit-identical to rr_kv_append followed by rr_extend_attention (with kRope, to the _rope pair).
 // kRope: q arrives un-rotated; as a unit's Q tiles land, each softmax thread rotates its own row at its
 // position P_b + i in shared memory, and the MMA issuer starts S_q only once tile q is rotated (the
 // keys were rotated on their way into the pool).
@@ -269,6 +381,8 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
     const Ctl ctl{abort_flag, a.err};
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    bool phase2 = true;
+    if constexpr (kFused) phase2 = fused_append<D, kRope>(a, *a.n_units, kNQ * a.tq);  // after the schedule kernel
 
     if (threadIdx.x == 0) {
         ptx::mbar_init(bar(C::kQFull), 1);
@@ -287,7 +401,6 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             ptx::mbar_init(bar(C::kOFinal + q), 1);
         }
         ptx::mbar_init(bar(C::kVTmp), 1);
-        ptx::mbar_init(bar(C::kKTmp), 1);
         for (int q = 0; q < kNQ; ++q) ptx::mbar_init(bar(C::kQRot + q), kBM);
         ptx::mbar_init(bar(C::kDrain), 1);
         ptx::mbar_init(bar(C::kDone), 2 * kBM);  // every softmax thread, once, at its end
@@ -302,17 +415,13 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
         ptx::prefetch_tmap(&a.tm_q);
         ptx::prefetch_tmap(&a.tm_k);
         ptx::prefetch_tmap(&a.tm_v);
-        if constexpr (kFused) {
-            ptx::prefetch_tmap(&a.tm_knew);
-            ptx::prefetch_tmap(&a.tm_vnew);
-        }
     }
     ptx::tc_fence_before();
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(smem + C::kOffMisc);
     ptx::griddep_wait();  // the schedule kernel's output (launched as its dependent)
-    const int n_units = kCas == kCasShared ? a.cas_units : *a.n_units;
+    const int n_units = !phase2 ? 0 : kCas == kCasShared ? a.cas_units : *a.n_units;
     const int grid = gridDim.x, cta = blockIdx.x;
     const int unit_tokens = kNQ * a.tq;
 
@@ -322,9 +431,9 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
     if (warp == kWarpProducer) {
         // ------------------------------------------------------------ TMA producer
         const int ppt = kBN / a.ps;  // pages per KV tile (<= 16)
-        uint32_t kv_count = 0, unit_i = 0, vtmp_phase = 0, ktmp_phase = 0;
+        uint32_t kv_count = 0, unit_i = 0, vtmp_phase = 0;
         // copies in flight, for the abort drain: bit s of armed_* = stage s armed, bit s of par_* = its parity
-        int armed_q = -1, armed_vtmp = -1, armed_ktmp = -1;
+        int armed_q = -1, armed_vtmp = -1;
         uint32_t armed_k = 0, armed_v = 0, par_k = 0, par_v = 0;
         bool ok = true;
         for (int w = 0; ok; ++w) {
@@ -363,48 +472,34 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             for (int j = kb; j < ke; ++j, ++kv_count) {
                 const int sk = (int)(kv_count % NK), sv = (int)(kv_count % NV);
                 const uint32_t usek = kv_count / NK, usev = kv_count / NV;
-                // the page of this lane: from the pool, from k_new / v_new (a fused step's suffix
-                // positions), or past the agent's keys (a row past the pool: zero fill)
+                // the page of this lane: from the pool, or past the agent's keys (a row past the pool: zero fill)
                 int row = a.oob_row;
-                bool from_new = false;
                 if (lane < ppt) {
                     const int lp = j * ppt + lane;
                     if (lp * a.ps < n_keys) {
-                        if (kFused && lp * a.ps >= P) {
-                            from_new = true;
-                            row = cu_b + (lp * a.ps - P);
-                        } else {
-                            const int pid = a.page_table[(long long)b * a.max_pages + lp];
-                            if (pid >= 0 && (long long)pid < a.num_pages) row = pid * a.ps;
-                            else atomicCAS(a.err, 0, RR_ERR_OOB);
-                        }
+                        const int pid = a.page_table[(long long)b * a.max_pages + lp];
+                        if (pid >= 0 && (long long)pid < a.num_pages) row = pid * a.ps;
+                        else atomicCAS(a.err, 0, RR_ERR_OOB);
                     }
                 }
-                // fused step, P in the middle of a page: that page comes from the pool and its slots
-                // from P on are rewritten from k_new / v_new in shared memory before the tiles are released
-                const bool straddle = kFused && (P % a.ps != 0) && (j == P / kBN);
                 // K tile
-                const uint32_t kbar = straddle ? bar(C::kKTmp) : bar(C::kKFull + sk);
+                const uint32_t kbar = bar(C::kKFull + sk);
                 if (lane == 0) {
                     if (usek > 0) ok = wait_bar(bar(C::kKEmpty + sk), (usek - 1) & 1, ctl);
                     if (ok) ptx::mbar_arrive_expect_tx(kbar, C::kKVTileBytes);
                 }
                 ok = __shfl_sync(0xffffffffu, ok, 0);
                 if (!ok) break;
-                if (!straddle) {
-                    armed_k |= 1u << sk;
-                    par_k = (par_k & ~(1u << sk)) | ((usek & 1u) << sk);
-                }
+                armed_k |= 1u << sk;
+                par_k = (par_k & ~(1u << sk)) | ((usek & 1u) << sk);
                 if (lane < ppt)
                     for (int c = 0; c < C::kChunks; ++c)
                         ptx::tma_load_2d(sb + C::kOffK + sk * C::kKVTileBytes + c * C::kChunkBytes + lane * a.ps * 128,
-                                         from_new ? &a.tm_knew : &a.tm_k, g * D + c * 64, row, kbar);
-                // V tile; if the agent's last page is only partly its own (unfused), land it on the side
-                // barrier, clear the foreign slots, then release it to the MMA warp.  (A fused step reads
-                // a partial last page from v_new, whose rows past the agent are other agents' finite
-                // values or zero fill, unless it is the straddling page, which is rewritten anyway.)
-                const bool clear_tail = !kFused && (j == n_kv - 1) && (last_page_end > agent_len);
-                const uint32_t vbar = (clear_tail || straddle) ? bar(C::kVTmp) : bar(C::kVFull + sv);
+                                         &a.tm_k, g * D + c * 64, row, kbar);
+                // V tile; if the agent's last page is only partly its own, land it on the side barrier, clear
+                // the foreign slots, then release it to the MMA warp
+                const bool clear_tail = (j == n_kv - 1) && (last_page_end > agent_len);
+                const uint32_t vbar = clear_tail ? bar(C::kVTmp) : bar(C::kVFull + sv);
                 if (lane == 0) {
                     if (usev > 0) ok = wait_bar(bar(C::kVEmpty + sv), (usev - 1) & 1, ctl);
                     if (ok) ptx::mbar_arrive_expect_tx(vbar, C::kKVTileBytes);
@@ -414,47 +509,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                 if (lane < ppt)
                     for (int c = 0; c < C::kChunks; ++c)
                         ptx::tma_load_2d(sb + C::kOffV + sv * C::kKVTileBytes + c * C::kChunkBytes + lane * a.ps * 128,
-                                         from_new ? &a.tm_vnew : &a.tm_v, g * D + c * 64, row, vbar);
-                if constexpr (kFused) {
-                    if (straddle) {
-                        // positions P .. end of P's page: rows r0 .. r1 of the tile, rewritten from the
-                        // agent's k_new / v_new rows (zeros past the agent's end), in the 128-byte swizzled
-                        // layout TMA wrote (16-byte unit u of row r sits at unit u ^ (r & 7))
-                        const int r0 = P - j * kBN, r1 = min(((P / a.ps) + 1) * a.ps - j * kBN, kBN);
-                        const int per_row = C::kChunks * 8;
-                        armed_ktmp = (int)ktmp_phase;
-                        armed_vtmp = (int)vtmp_phase;
-                        for (int kv = 0; kv < 2 && ok; ++kv) {
-                            const uint32_t tb = kv == 0 ? bar(C::kKTmp) : bar(C::kVTmp);
-                            if (lane == 0) ok = wait_bar(tb, kv == 0 ? ktmp_phase : vtmp_phase, ctl);
-                            ok = __shfl_sync(0xffffffffu, ok, 0);
-                            if (!ok) break;
-                            if (kv == 0) {
-                                armed_ktmp = -1;
-                                ktmp_phase ^= 1u;
-                            } else {
-                                armed_vtmp = -1;
-                                vtmp_phase ^= 1u;
-                            }
-                            uint8_t* tile = smem + (kv == 0 ? C::kOffK + sk * C::kKVTileBytes
-                                                            : C::kOffV + sv * C::kKVTileBytes);
-                            const uint4* src = kv == 0 ? a.knew : a.vnew;
-                            for (int e = lane; e < (r1 - r0) * per_row; e += 32) {
-                                const int r = r0 + e / per_row, c = (e / 8) % C::kChunks, v = e % 8;
-                                const int pos = j * kBN + r;
-                                uint4 val = make_uint4(0u, 0u, 0u, 0u);
-                                if (pos < agent_len)
-                                    val = src[(long long)(cu_b + pos - P) * a.row16 + (g * D + c * 64) / 8 + v];
-                                *reinterpret_cast<uint4*>(tile + c * C::kChunkBytes + r * 128 + ((v ^ (r & 7)) << 4)) = val;
-                            }
-                            ptx::fence_proxy_async_smem();
-                            __syncwarp();
-                            if (lane == 0) ptx::mbar_arrive(kv == 0 ? bar(C::kKFull + sk) : bar(C::kVFull + sv));
-                        }
-                        if (!ok) break;
-                        continue;
-                    }
-                }
+                                         &a.tm_v, g * D + c * 64, row, vbar);
                 if (clear_tail) {
                     armed_vtmp = (int)vtmp_phase;
                     if (lane == 0) ok = wait_bar(bar(C::kVTmp), vtmp_phase, ctl);
@@ -481,7 +536,6 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
         if (!ok && lane == 0) {  // abort: let every copy this warp started land before exit
             if (armed_q >= 0) drain_bar(bar(C::kQFull), (uint32_t)armed_q);
             if (armed_vtmp >= 0) drain_bar(bar(C::kVTmp), (uint32_t)armed_vtmp);
-            if (armed_ktmp >= 0) drain_bar(bar(C::kKTmp), (uint32_t)armed_ktmp);
             for (int s = 0; s < NK; ++s)
                 if (armed_k >> s & 1u) drain_bar(bar(C::kKFull + s), par_k >> s & 1u);
             for (int s = 0; s < NV; ++s)
@@ -639,47 +693,6 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
         __syncwarp();
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem, 512);
-    } else if (kFused && warp == kWarpAppend) {
-        // ------------------------------------------------------------ pool writer (fused step)
-        // Each work unit's own suffix rows of its KV head go to the agent's pool slots (every (token,
-        // KV head) belongs to exactly one unit; one piece of a split unit writes).  The kernel reads
-        // suffix K/V from k_new / v_new, so nothing waits for these writes: they are for later calls.
-        // Two tokens per pass (16 lanes each at D = 128, 8 at D = 64: one 16-byte vector of K and one
-        // of V per lane), page and slot by shifts (page sizes are powers of two): the loop stays
-        // light, since this warp shares its scheduler with two softmax warps.
-        constexpr int kPerTok = D / 8;      // 16-byte vectors of one head's row
-        constexpr int kTokPerPass = 32 / kPerTok;
-        const int ps_shift = __ffs(a.ps) - 1;
-        const int sub = lane / kPerTok, v = lane % kPerTok;
-        for (int w = 0;; ++w) {
-            const int ui = unit_of(w, cta, grid);
-            if (ui >= n_units) break;
-            const int4 U = a.units[ui];
-            if (((U.y >> 8) & 0xFF) != 0) continue;
-            const int b = U.x, g = U.y & 0xFF, u = U.z;
-            const int P = a.prefix[b], S = a.suffix[b], cu_b = a.cu[b];
-            const int t0 = u * unit_tokens, n = min(unit_tokens, S - t0);
-            const int32_t* pt = a.page_table + (long long)b * a.max_pages;
-            for (int tt = 0; tt < n; tt += kTokPerPass) {
-                const int t = tt + sub;
-                if (t >= n) continue;
-                const int pos = P + t0 + t;
-                const int pid = pt[pos >> ps_shift];
-                if (pid < 0 || (long long)pid >= a.num_pages) {
-                    atomicCAS(a.err, 0, RR_ERR_OOB);
-                    continue;
-                }
-                const long long src = (long long)(cu_b + t0 + t) * a.row16 + g * kPerTok + v;
-                const long long dst = (((long long)pid << ps_shift) + (pos & (a.ps - 1))) * a.row16 + g * kPerTok + v;
-                // streaming (evict-first) on both sides: nothing in this launch reads these lines again, and
-                // with default-policy stores the 2 x T x Hkv x D x 2 bytes pushed the units' shared K/V out of
-                // L2 (measured: 5 % of the step on c2, c4 and c5)
-                const uint4 kx = __ldcs(a.knew + src);
-                const uint4 vx = __ldcs(a.vnew + src);
-                __stcs(a.kpool + dst, kx);
-                __stcs(a.vpool + dst, vx);
-            }
-        }
     }
     return;
     }
@@ -974,6 +987,20 @@ cudaError_t launch_cfg(const AttnArgs& a, int grid, cudaStream_t st) {
     if constexpr (kCas == kCasShared) {  // needs no schedule: an ordinary launch
         extend_attn_kernel<D, NK, NV, kFused, kRope, kCas><<<grid, kThreads, C::kSmemBytes, st>>>(a);
         return cudaGetLastError();
+    } else if constexpr (kFused) {
+        // the grid barrier between the two phases needs every CTA resident: a cooperative launch (the
+        // runtime refuses a grid larger than the device holds), started once the schedule has finished
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(grid);
+        cfg.blockDim = dim3(kThreads);
+        cfg.dynamicSmemBytes = C::kSmemBytes;
+        cfg.stream = st;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeCooperative;
+        attr[0].val.cooperative = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        return cudaLaunchKernelEx(&cfg, extend_attn_kernel<D, NK, NV, kFused, kRope, kCas>, a);
     } else {
         return launch_after_sched(extend_attn_kernel<D, NK, NV, kFused, kRope, kCas>, dim3(grid), dim3(kThreads),
                                   C::kSmemBytes, st, a);
@@ -999,13 +1026,13 @@ cudaError_t launch_extend_cascade(const AttnArgs& a, int head_dim, int grid, cud
 }
 
 cudaError_t launch_extend_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st, bool fused) {
-    if (fused && a.rope) return cudaErrorInvalidValue;  // the one-launch step takes rotated rows only
+    if (fused && !a.grid_sync) return cudaErrorInvalidValue;
     if (head_dim == 128) {
-        if (fused) return launch_cfg<128, 2, 3, true, false>(a, grid, st);
+        if (fused) return a.rope ? launch_cfg<128, 2, 3, true, true>(a, grid, st) : launch_cfg<128, 2, 3, true, false>(a, grid, st);
         return a.rope ? launch_cfg<128, 2, 3, false, true>(a, grid, st) : launch_cfg<128, 2, 3, false, false>(a, grid, st);
     }
     if (head_dim == 64) {
-        if (fused) return launch_cfg<64, 4, 4, true, false>(a, grid, st);
+        if (fused) return a.rope ? launch_cfg<64, 4, 4, true, true>(a, grid, st) : launch_cfg<64, 4, 4, true, false>(a, grid, st);
         return a.rope ? launch_cfg<64, 4, 4, false, true>(a, grid, st) : launch_cfg<64, 4, 4, false, false>(a, grid, st);
     }
     return cudaErrorInvalidValue;

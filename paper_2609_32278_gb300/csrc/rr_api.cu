@@ -189,8 +189,8 @@ namespace {
 
 // Extend attention; decode attention (decode = true: kv_lens in place of the prefix / suffix lengths,
 // one query token per agent, the decode kernel in place of the extend kernel); or the fused extend
-// step (k_new / v_new non-null: the extend kernel reads the suffix K/V from them and writes them into
-// the pools itself).
+// step (k_new / v_new non-null: the extend kernel first writes them into the pools, rotating K when a
+// rope table is given, then attends over the pools).
 int attention_impl(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,
                    const int32_t* prefix_lens, const int32_t* suffix_lens, const int32_t* kv_lens, void* out,
                    const rr_dims* dims, float softmax_scale, cudaStream_t stream, bool decode,
@@ -204,7 +204,6 @@ int attention_impl(const void* q, const void* k_pool, const void* v_pool, const 
     if (rope && dims->total_tokens > 0) {
         if (!aligned16(rope)) return fail(RR_ERR_INVALID_ARG, "rope table must be 16-byte aligned");
         if (rope_max_pos <= 0) return fail(RR_ERR_INVALID_ARG, "rope_max_pos must be positive");
-        if (fused) return fail(RR_ERR_UNSUPPORTED, "the one-launch extend step takes rotated rows only");
     }
     if (fused) {
         if (!k_new || !v_new) return fail(RR_ERR_INVALID_ARG, "the fused step needs both k_new and v_new");
@@ -283,6 +282,7 @@ int attention_impl(const void* q, const void* k_pool, const void* v_pool, const 
     s.split_waves = split_waves;
     s.n_units = reinterpret_cast<int32_t*>(ws);
     s.lens_ok = reinterpret_cast<int32_t*>(ws) + 1;
+    if (fused) s.grid_sync = reinterpret_cast<int32_t*>(ws) + 3;
     s.err = d->err;
     e = rr::launch_sched(s, stream);
     if (e != cudaSuccess) return cuda_fail(e, "schedule kernel launch");
@@ -322,10 +322,9 @@ int attention_impl(const void* q, const void* k_pool, const void* v_pool, const 
     a.wait_hint_ns = (uint32_t)std::min<long long>(200000, std::max<long long>(1, a.wait_limit / 4));
     const int64_t grid = std::min<int64_t>((int64_t)d->sm_count, max_items);
     if (fused) {
-        // k_new / v_new [T][Hkv][D]: one row of Hkv * D per suffix token, the pool maps' box
+        // k_new / v_new [T][Hkv][D]: one row of Hkv * D per suffix token
         const uint64_t row_elems = (uint64_t)Hkv * D;
-        if ((rc = encode_2d(&a.tm_knew, k_new, row_elems, (uint64_t)T, row_elems * 2, 64, (uint32_t)ps))) return rc;
-        if ((rc = encode_2d(&a.tm_vnew, v_new, row_elems, (uint64_t)T, row_elems * 2, 64, (uint32_t)ps))) return rc;
+        a.grid_sync = s.grid_sync;
         a.knew = static_cast<const uint4*>(k_new);
         a.vnew = static_cast<const uint4*>(v_new);
         a.kpool = static_cast<uint4*>(const_cast<void*>(k_pool));
@@ -767,11 +766,10 @@ int rr_extend_step_rope(const void* q, const void* k_new, const void* v_new, voi
                         const rr_dims* dims, float softmax_scale, const float* rope_table, int32_t rope_max_pos,
                         cudaStream_t stream) {
     if (!rope_table) return fail(RR_ERR_INVALID_ARG, "null rope table");
-    int rc = append_impl(k_new, v_new, k_pool, v_pool, page_table, prefix_lens, suffix_lens, dims, stream, rope_table,
-                         rope_max_pos);
-    if (rc) return rc;
+    const bool any = dims && dims->total_tokens > 0;
+    if (any && (!k_new || !v_new)) return fail(RR_ERR_INVALID_ARG, "null k_new / v_new");
     return attention_impl(q, k_pool, v_pool, page_table, prefix_lens, suffix_lens, nullptr, out, dims, softmax_scale,
-                          stream, false, nullptr, nullptr, rope_table, rope_max_pos);
+                          stream, false, any ? k_new : nullptr, any ? v_new : nullptr, rope_table, rope_max_pos);
 }
 
 int rr_extend_attention(const void* q, const void* k_pool, const void* v_pool, const int32_t* page_table,

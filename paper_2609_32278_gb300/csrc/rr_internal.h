@@ -51,6 +51,7 @@ struct SchedArgs {
     int32_t min_prefix;    // every agent's prefix must be at least this long (extend over a shared prefix)
     int32_t* n_units;      // number of items
     int32_t* lens_ok;
+    int32_t* grid_sync;    // set to 0 (the fused extend step's grid-barrier counter), if non-null
     int32_t* err;
 };
 
@@ -97,9 +98,9 @@ struct AttnArgs {
     long long wait_limit;  // cycles a pipeline wait may take before the kernel gives up (RR_ERR_TIMEOUT):
                            // every wait of the decode kernel, the extend kernel's stage watcher
     uint32_t wait_hint_ns; // how long one try of such a wait may suspend the thread
-    // fused extend step only (the suffix K/V is read from k_new / v_new and written to the pool here)
-    CUtensorMap tm_knew;   // k_new [T][Hkv*D], box {64, ps}, 128B swizzle
-    CUtensorMap tm_vnew;   // v_new, same
+    // fused extend step only: the kernel first writes k_new / v_new into the pool (K rotated when rope is
+    // set), then crosses a grid barrier on grid_sync (zeroed by the schedule kernel) before the attention
+    int32_t* grid_sync;
     const uint4* knew;     // k_new / v_new rows and pool rows, 16-byte vectors
     const uint4* vnew;
     uint4* kpool;
@@ -164,8 +165,9 @@ cudaError_t launch_sched(const SchedArgs& a, cudaStream_t st);
 cudaError_t launch_combine(const CombineArgs& a, int grid, cudaStream_t st);
 cudaError_t launch_kv_append(const AppendArgs& a, int sm_count, cudaStream_t st);
 // Returns cudaErrorInvalidValue for an unsupported head dim.  fused: the one-launch extend step (the
-// suffix K/V come from k_new / v_new, and the kernel also writes them into the pool).  a.rope set: q
-// is rotated in shared memory as each Q tile lands (not with fused).
+// kernel writes k_new / v_new into the pool, waits at a grid barrier on a.grid_sync, then attends over
+// the pool; a cooperative launch).  a.rope set: q is rotated in shared memory as each Q tile lands (and,
+// fused, each K row on its way into the pool).
 cudaError_t launch_extend_attention(const AttnArgs& a, int head_dim, int grid, cudaStream_t st, bool fused = false);
 // The two passes of rr_extend_attention_shared (shared_pass: every suffix row against the shared keys, an
 // ordinary launch; otherwise the schedule's units over the private keys, merging, as the schedule's dependent).

@@ -101,7 +101,10 @@ __global__ void __launch_bounds__(1024) sched_kernel(SchedArgs a) {
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     // the consumer kernel may start its prologue now; it waits for this kernel before reading its output
     ptx::griddep_launch_dependents();
-    if (tid == 0) s_bad = 0;
+    if (tid == 0) {
+        s_bad = 0;
+        if (a.grid_sync) *a.grid_sync = 0;
+    }
     __syncthreads();
 
     // ---- 1. validate, per-thread sums over a contiguous chunk of agents

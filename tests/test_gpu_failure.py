@@ -1,7 +1,7 @@
 """The bounded-wait failure path of the attention kernels, provoked without a GPU fault.
 
 rr_set_wait_limit shortens the budget of the kernels' pipeline waits (every wait of the decode kernel,
-the stage watcher's in the extend kernel), and with it how long one try may suspend the thread, to a
+the stage watcher's in the extend kernel, the one-launch step's grid barrier), and with it how long one try may suspend the thread, to a
 few hundred clock cycles, far below a tile's load time, so the first such wait runs out.  Each such call must end with RR_ERR_TIMEOUT in the device error word -- every role leaves its
 loop, copies and tensor-core operations in flight are drained, tensor memory is freed -- and the context
 must stay usable: with the default budget restored, the same call returns, bit for bit, what it returned

@@ -1,8 +1,12 @@
-"""The fused extend step (rr_extend_step): append + attention in one attention launch.
+"""The fused extend step (rr_extend_step, rr_extend_step_rope): append + attention in one launch.
 
-Checked three ways on the same seeded inputs: the pools bit-exact against the oracle's append,
+The kernel writes every suffix row into the pool, crosses a grid barrier, then attends over the pool;
+its first phase hands rows out over all warps of the grid, its second runs the schedule's units, so
+nearly every unit reads suffix rows another CTA wrote (the barrier's ordering is under test in every
+case).  Checked three ways on the same seeded inputs: the pools bit-exact against the oracle's append,
 the output against the fp64 oracle within the parity bar, and the output bit-identical to
-rr_kv_append followed by rr_extend_attention (the same arithmetic on the same values).  Cases
+rr_kv_append followed by rr_extend_attention (the same arithmetic on the same values); with a rotary
+table, pools and output bit-identical to rr_kv_append_rope followed by rr_extend_attention_rope.  Cases
 cover prefixes in the middle of a page (the page holding both cached and new positions),
 page-aligned prefixes, no prefix, one-token suffixes, agents without suffix, every GQA group,
 both head dims and split-K batches (one writer per split unit).
@@ -129,3 +133,43 @@ def test_fused_step_reports_bad_page(rr):
     with pytest.raises(ValueError):
         rr.extend_step(g["q"], g["k_new"][:10], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"],
                        g["prefix_lens"], g["suffix_lens"])
+
+
+ROPE_BASE = 500000.0
+
+
+@pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
+def test_fused_rope_step_equals_its_two_calls(rr, case):
+    name, B, Hq, Hkv, D, P, S = case
+    wl = synth.custom(name, B, Hq, Hkv, D, P, S, seed=7)
+    table = rr.rope_table(int(max(np.asarray(P) + np.asarray(S))) + 1, D, ROPE_BASE)
+    g1 = synth.gpu_tensors(wl, "cuda")
+    rr.kv_append(g1["k_new"], g1["v_new"], g1["k_pool"], g1["v_pool"], g1["page_table"], g1["prefix_lens"],
+                 g1["suffix_lens"], rope=table)
+    out1 = rr.extend_attention(g1["q"], g1["k_pool"], g1["v_pool"], g1["page_table"], g1["prefix_lens"],
+                               g1["suffix_lens"], rope=table)
+    assert rr.device_error() == 0, rr.last_error()
+    g2 = synth.gpu_tensors(wl, "cuda")
+    out2 = rr.extend_step(g2["q"], g2["k_new"], g2["v_new"], g2["k_pool"], g2["v_pool"], g2["page_table"],
+                          g2["prefix_lens"], g2["suffix_lens"], rope=table)
+    assert rr.device_error() == 0, rr.last_error()
+    np.testing.assert_array_equal(u16(g1["k_pool"]), u16(g2["k_pool"]))
+    np.testing.assert_array_equal(u16(g1["v_pool"]), u16(g2["v_pool"]))
+    np.testing.assert_array_equal(bf16_bits(out1), bf16_bits(out2))
+
+
+def test_fused_rope_step_position_past_table_is_reported(rr):
+    wl = synth.custom("short_table_step", 2, 8, 2, 128, [100, 10], [20, 5], seed=17)
+    g = synth.gpu_tensors(wl, "cuda")
+    table = rr.rope_table(110, 128, ROPE_BASE)  # agent 0 reaches position 119
+    rr.extend_step(g["q"], g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                   g["suffix_lens"], rope=table)
+    assert rr.device_error() == rr.RR_ERR_LENS
+    # the rows it could rotate are in the pool exactly as the separate rotated append leaves them (rows past
+    # the table are written by neither)
+    g2 = synth.gpu_tensors(wl, "cuda")
+    rr.kv_append(g2["k_new"], g2["v_new"], g2["k_pool"], g2["v_pool"], g2["page_table"], g2["prefix_lens"],
+                 g2["suffix_lens"], rope=table)
+    assert rr.device_error() == rr.RR_ERR_LENS
+    np.testing.assert_array_equal(u16(g["k_pool"]), u16(g2["k_pool"]))
+    np.testing.assert_array_equal(u16(g["v_pool"]), u16(g2["v_pool"]))
