@@ -86,6 +86,20 @@ def load_peaks():
         return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
 
 
+# The measured bf16 peaks come as a burst (best of ten 8192^3 GEMMs) and as a sustained figure (the same GEMM
+# back to back for 4 s under the power cap).  A tensor-bound kernel is held to the one that matches how long its
+# timed loop runs back to back: the burst under a second, the sustained beyond.
+SUSTAINED_AFTER_MS = 1000.0
+
+
+def tensor_peak(peaks, timed_ms):
+    """(peak TFLOP/s, description) for a tensor-bound kernel whose timed loop ran `timed_ms` back to back."""
+    if timed_ms >= SUSTAINED_AFTER_MS:
+        return peaks["bf16_sus"], (f"{peaks['src']} bf16 dense sustained (the timed loop runs {timed_ms / 1e3:.1f} s "
+                                   f"back to back, the regime the sustained GEMM figure was taken in)")
+    return peaks["bf16"], f"{peaks['src']} bf16 dense burst (the timed loop runs {timed_ms:.0f} ms)"
+
+
 class ClockSampler:
     """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
 
@@ -361,13 +375,15 @@ def config_leg(rr, synth, name, steps, warmup, dev, st, peaks, rank, local):
     attn_ms = statistics.mean(e1.elapsed_time(e2) for e0, e1, e2 in ev)
     app_ms = statistics.mean(e0.elapsed_time(e1) for e0, e1, e2 in ev)
     achieved = F / (attn_ms * 1e-3) / 1e12
+    leg_peak, leg_kind = tensor_peak(peaks, steps * step_ms)
     res = {"config": config_dict(wl, 1), "inputs_sha256": wl.manifest()["sha256"][:16], "steps": steps,
            "warmup": warmup, "ms_per_step": step_ms, "value": F / (step_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
            "uncached_suffix_tokens_per_s": wl.T / (step_ms * 1e-3), "attention_ms": attn_ms,
            "attention_ms_median": statistics.median(e1.elapsed_time(e2) for e0, e1, e2 in ev),
            "kv_append_ms": app_ms, "kv_append_gbs": append_bytes(wl) / (app_ms * 1e-3) / 1e9,
-           "roofline": {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16"], "unit": "TFLOP/s",
-                        "frac": achieved / peaks["bf16"], "frac_of_sustained": achieved / peaks["bf16_sus"],
+           "roofline": {"bound": "tensor", "achieved": achieved, "peak": leg_peak, "unit": "TFLOP/s",
+                        "frac": achieved / leg_peak, "peak_kind": leg_kind, "frac_of_burst": achieved / peaks["bf16"],
+                        "frac_of_sustained": achieved / peaks["bf16_sus"],
                         "frac_of_nominal": achieved / NOMINAL_BF16_TFLOPS,
                         "traffic": traffic_for(wl.name, kernel_source_hash()),
                         "algorithmic_flops": F, "algorithmic_bytes": attn_bytes(wl)},
@@ -840,10 +856,11 @@ def run_ours(args, world, rank, local):
     achieved = F / (attn_ms * 1e-3) / 1e12
     src_hash = kernel_source_hash()
     traffic = traffic_for(wl.name, src_hash)  # recorded for this whole batch (scaled from a slice), or None
-    roof = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16"], "unit": "TFLOP/s",
-            "frac": achieved / peaks["bf16"], "traffic": traffic,
-            "peak_kind": f"{peaks['src']} bf16 dense burst (the timed loop is well under a second)",
-            "frac_of_sustained": achieved / peaks["bf16_sus"], "frac_of_nominal": achieved / NOMINAL_BF16_TFLOPS,
+    peak, peak_kind = tensor_peak(peaks, args.steps * ms_step)
+    roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+            "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
+            "frac_of_burst": achieved / peaks["bf16"], "frac_of_sustained": achieved / peaks["bf16_sus"],
+            "frac_of_nominal": achieved / NOMINAL_BF16_TFLOPS,
             "kernel": "extend_attn_kernel<128,2,3>" if wl.D == 128 else "extend_attn_kernel<64,4,4>",
             "algorithmic_bytes": attn_bytes(wl), "algorithmic_flops": F,
             "bytes_bound_frac": attn_bytes(wl) / (attn_ms * 1e-3) / 1e9 / peaks["hbm"],

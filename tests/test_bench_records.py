@@ -90,3 +90,18 @@ def test_policy_pair_workloads():
     if os.path.exists(rr._SO):
         for w in (a, b):
             assert rr.validate_page_table(w.page_table, w.prefix_lens, w.suffix_lens, w.num_pages, w.ps) == 0
+
+
+def test_tensor_peak_follows_the_timed_loop_length():
+    """A timed loop of a second or more runs in the power-capped regime of the sustained GEMM figure; a shorter
+    one is held to the burst figure.  Both are the measured numbers, never a mix."""
+    peaks = dict(hbm=6685.8, bf16=1881.8, bf16_sus=1741.7, src="measured")
+    p, kind = bench.tensor_peak(peaks, 190.0)          # c2: 20 steps of ~9.5 ms
+    assert p == 1881.8 and "burst" in kind
+    p, kind = bench.tensor_peak(peaks, 20 * 213.0)     # c4: 20 steps of ~213 ms
+    assert p == 1741.7 and "sustained" in kind
+    p, _ = bench.tensor_peak(peaks, bench.SUSTAINED_AFTER_MS)
+    assert p == 1741.7
+    fb = dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
+    p, kind = bench.tensor_peak(fb, 5000.0)
+    assert p == 1700.0 and kind.startswith("fallback")
