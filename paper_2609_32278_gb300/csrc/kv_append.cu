@@ -13,6 +13,9 @@
 // (streaming loads); the pool writes keep the default policy because the
 // attention kernel reads those pages right after.
 //
+// Batches of up to kAppendSelfLensMaxB agents run as this one kernel: every block checks the lengths and takes
+// the suffix prefix sums itself (self_lens), which takes the schedule kernel and its launch off the call.
+//
 // With a rotary table (kRope), each K row is rotated at its position P_b + j
 // on the way into the pool (rope.cuh): a lane takes the two 16-byte vectors of
 // one head that hold a rotation pair's halves (dims i0.. and i0 + D/2..), so
@@ -37,19 +40,73 @@ __device__ __forceinline__ int last_le(const int32_t* off, int n, long long x) {
 
 constexpr int kAppendThreads = 256;
 constexpr int kCuSmem = 2048;  // agents whose suffix prefix sums a block stages in shared memory
+static_assert(kAppendSelfLensMaxB < kCuSmem, "the self-checking path keeps B + 1 prefix sums in shared memory");
+
+// The schedule kernel's length check and prefix sums, done by one block for itself (batches of fewer than
+// kCuSmem agents): each thread takes a contiguous run of agents, checks 0 <= P, 0 <= S, P + S <= the page
+// table's capacity, and the block scans the suffix lengths into s_cu[0..B]; the sum must equal T.  Every block
+// reaches the same verdict from the same lengths; block 0 reports a bad batch (RR_ERR_LENS) and no block writes.
+__device__ bool self_lens(const AppendArgs& a, int32_t* s_cu) {
+    __shared__ long long s_w[kAppendThreads / 32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int B = a.B;
+    const int per = (B + kAppendThreads - 1) / kAppendThreads;
+    const int b0 = min(B, (int)threadIdx.x * per), b1 = min(B, b0 + per);
+    const long long cap = (long long)a.max_pages * a.ps;
+    long long sum = 0;
+    bool bad = false;
+    for (int b = b0; b < b1; ++b) {
+        const int P = a.prefix[b], S = a.suffix[b];
+        if (P < 0 || S < 0 || (long long)P + S > cap) bad = true;
+        sum += S;
+    }
+    long long inc = sum;  // inclusive scan over the block, in thread order
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const long long y = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += y;
+    }
+    if (lane == 31) s_w[warp] = inc;
+    __syncthreads();
+    long long before = 0, total = 0;
+#pragma unroll
+    for (int w = 0; w < kAppendThreads / 32; ++w) {
+        if (w < warp) before += s_w[w];
+        total += s_w[w];
+    }
+    long long off = before + inc - sum;
+    const bool ok = !__syncthreads_or(bad) && total == a.T && total < (1ll << 31);
+    if (!ok) {
+        if (blockIdx.x == 0 && threadIdx.x == 0) atomicCAS(a.err, 0, RR_ERR_LENS);
+        return false;
+    }
+    for (int b = b0; b < b1; ++b) {
+        s_cu[b] = (int32_t)off;
+        off += a.suffix[b];
+    }
+    if (threadIdx.x == 0) s_cu[B] = (int32_t)total;
+    __syncthreads();
+    return true;
+}
 
 
-template <bool kRope>
+// kSelf: the lengths are checked and summed by the kernel itself (self_lens) instead of by the schedule kernel.
+template <bool kRope, bool kSelf>
 __global__ void __launch_bounds__(kAppendThreads) kv_append_kernel(const AppendArgs a) {
     __shared__ int32_t s_cu[kCuSmem];
-    ptx::griddep_wait();  // the schedule kernel's output (launched as its dependent)
-    if (*a.lens_ok == 0) return;
     // each token's agent is a binary search over the suffix prefix sums: from shared memory when they fit,
     // so a token's copy does not wait behind log2(B) dependent global loads
-    const bool cu_in_smem = a.B < kCuSmem;
-    if (cu_in_smem) {
-        for (int i = threadIdx.x; i <= a.B; i += kAppendThreads) s_cu[i] = a.cu[i];
-        __syncthreads();
+    bool cu_in_smem = true;
+    if constexpr (kSelf) {
+        if (!self_lens(a, s_cu)) return;
+    } else {
+        ptx::griddep_wait();  // the schedule kernel's output (launched as its dependent)
+        if (*a.lens_ok == 0) return;
+        cu_in_smem = a.B < kCuSmem;
+        if (cu_in_smem) {
+            for (int i = threadIdx.x; i <= a.B; i += kAppendThreads) s_cu[i] = a.cu[i];
+            __syncthreads();
+        }
     }
     const int32_t* __restrict__ cu = cu_in_smem ? s_cu : a.cu;
     const int lane = threadIdx.x & 31;
@@ -120,8 +177,13 @@ cudaError_t launch_kv_append(const AppendArgs& a, int sm_count, cudaStream_t st)
     const long long cap = (long long)sm_count * 8;  // 8 resident blocks of 256 threads per SM
     if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
-    cudaError_t e = a.rope ? launch_after_sched(kv_append_kernel<true>, dim3((unsigned)blocks), dim3(kAppendThreads), 0, st, a)
-                           : launch_after_sched(kv_append_kernel<false>, dim3((unsigned)blocks), dim3(kAppendThreads), 0, st, a);
+    if (a.self_lens) {  // an ordinary launch: it runs once the kernels before it on the stream have finished
+        if (a.rope) kv_append_kernel<true, true><<<(unsigned)blocks, kAppendThreads, 0, st>>>(a);
+        else kv_append_kernel<false, true><<<(unsigned)blocks, kAppendThreads, 0, st>>>(a);
+        return cudaGetLastError();
+    }
+    cudaError_t e = a.rope ? launch_after_sched(kv_append_kernel<true, false>, dim3((unsigned)blocks), dim3(kAppendThreads), 0, st, a)
+                           : launch_after_sched(kv_append_kernel<false, false>, dim3((unsigned)blocks), dim3(kAppendThreads), 0, st, a);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }

@@ -664,6 +664,34 @@ int append_impl(const void* k_new, const void* v_new, void* k_pool, void* v_pool
         return fail(RR_ERR_INVALID_ARG, "int32 arrays must be 4-byte aligned");
     Device* d = nullptr;
     if ((rc = current_device(&d, nullptr))) return rc;
+    rr::AppendArgs a{};
+    a.k_new = static_cast<const uint4*>(k_new);
+    a.v_new = static_cast<const uint4*>(v_new);
+    a.k_pool = static_cast<uint4*>(k_pool);
+    a.v_pool = static_cast<uint4*>(v_pool);
+    a.page_table = page_table;
+    a.prefix = prefix_lens;
+    a.suffix = suffix_lens;
+    a.err = d->err;
+    a.T = dims->total_tokens;
+    a.num_pages = dims->num_pages;
+    a.B = dims->batch;
+    a.max_pages = dims->max_pages;
+    a.ps = dims->page_size;
+    a.row16 = dims->num_kv_heads * dims->head_dim * 2 / 16;
+    if (rope) {
+        a.rope = reinterpret_cast<const float2*>(rope);
+        a.rope_max_pos = rope_max_pos;
+        a.hkv = dims->num_kv_heads;
+        a.d16 = dims->head_dim / 16;
+    }
+    cudaError_t e = cudaSuccess;
+    if (dims->batch <= rr::kAppendSelfLensMaxB) {  // one kernel: it checks and sums the lengths itself
+        a.self_lens = 1;
+        e = rr::launch_kv_append(a, d->sm_count, stream);
+        if (e != cudaSuccess) return cuda_fail(e, "kv_append kernel launch");
+        return RR_OK;
+    }
     const Layout L = layout_for(dims->batch, 0);
     if ((rc = ensure_ws(*d, L.total))) return rc;
     uint8_t* ws = static_cast<uint8_t*>(d->ws);
@@ -689,32 +717,12 @@ int append_impl(const void* k_new, const void* v_new, void* k_pool, void* v_pool
     s.n_units = reinterpret_cast<int32_t*>(ws);
     s.lens_ok = reinterpret_cast<int32_t*>(ws) + 1;
     s.err = d->err;
-    cudaError_t e = rr::launch_sched(s, stream);
+    e = rr::launch_sched(s, stream);
     if (e != cudaSuccess) return cuda_fail(e, "schedule kernel launch");
     if (dims->total_tokens == 0) return RR_OK;
 
-    rr::AppendArgs a{};
-    a.k_new = static_cast<const uint4*>(k_new);
-    a.v_new = static_cast<const uint4*>(v_new);
-    a.k_pool = static_cast<uint4*>(k_pool);
-    a.v_pool = static_cast<uint4*>(v_pool);
-    a.page_table = page_table;
-    a.prefix = prefix_lens;
     a.cu = s.cu;
     a.lens_ok = s.lens_ok;
-    a.err = d->err;
-    a.T = dims->total_tokens;
-    a.num_pages = dims->num_pages;
-    a.B = dims->batch;
-    a.max_pages = dims->max_pages;
-    a.ps = dims->page_size;
-    a.row16 = dims->num_kv_heads * dims->head_dim * 2 / 16;
-    if (rope) {
-        a.rope = reinterpret_cast<const float2*>(rope);
-        a.rope_max_pos = rope_max_pos;
-        a.hkv = dims->num_kv_heads;
-        a.d16 = dims->head_dim / 16;
-    }
     e = rr::launch_kv_append(a, d->sm_count, stream);
     if (e != cudaSuccess) return cuda_fail(e, "kv_append kernel launch");
     return RR_OK;

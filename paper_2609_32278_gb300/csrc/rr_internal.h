@@ -62,6 +62,7 @@ struct AppendArgs {
     uint4* v_pool;
     const int32_t* page_table;
     const int32_t* prefix;
+    const int32_t* suffix;     // read only when the kernel checks the lengths itself (self_lens)
     const int32_t* cu;
     const int32_t* lens_ok;
     int32_t* err;
@@ -73,7 +74,11 @@ struct AppendArgs {
     const float2* rope;
     int32_t rope_max_pos;
     int32_t hkv, d16;      // KV heads; D / 16 = rotation pair vectors per head
+    // batches of at most kAppendSelfLensMaxB agents: the append kernel checks the lengths and takes the suffix
+    // prefix sums itself, in every block, and runs without the schedule kernel in front of it
+    int32_t self_lens;
 };
+constexpr int kAppendSelfLensMaxB = 2047;
 
 struct AttnArgs {
     CUtensorMap tm_q;      // q   [T][Hq][D]        box {64, G, 128/G}, 128B swizzle

@@ -121,3 +121,33 @@ def test_append_rejects_bad_arguments(rr):
         rr.kv_append(g["k_new"][:, :1], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
                      g["suffix_lens"])
     del torch
+
+
+@pytest.mark.parametrize("B", [2047, 2048, 3001])
+def test_append_bit_exact_many_agents(rr, B):
+    """Up to 2047 agents the append kernel checks and sums the lengths itself; beyond, the schedule kernel does it
+    first.  Both sides of the switch, mid-page prefixes and empty suffixes among them, land bit-exact."""
+    rng = np.random.default_rng(B)
+    P = rng.integers(0, 40, size=B)
+    S = rng.integers(0, 4, size=B)
+    wl = synth.custom(f"many_{B}", B, 4, 2, 64, P, S, seed=9)
+    g, code = _run(rr, wl)
+    assert code == 0
+    kp, vp = _expected(wl)
+    np.testing.assert_array_equal(bf16_bits(g["k_pool"]), kp)
+    np.testing.assert_array_equal(bf16_bits(g["v_pool"]), vp)
+
+
+@pytest.mark.parametrize("B", [2, 2100])
+def test_append_negative_prefix_is_a_device_error(rr, B):
+    """A negative cached length fails the check on either path: RR_ERR_LENS, nothing written."""
+    P = np.full(B, 16, dtype=np.int64)
+    S = np.full(B, 2, dtype=np.int64)
+    wl = synth.custom(f"negp_{B}", B, 4, 2, 64, P, S, seed=3)
+    g = synth.gpu_tensors(wl, "cuda", pool_fill=0x1357)
+    before = bf16_bits(g["k_pool"]).copy()
+    pl = g["prefix_lens"].clone()
+    pl[B - 1] = -1
+    rr.kv_append(g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], pl, g["suffix_lens"])
+    assert rr.device_error() == rr.RR_ERR_LENS
+    np.testing.assert_array_equal(bf16_bits(g["k_pool"]), before)
