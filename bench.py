@@ -880,7 +880,8 @@ def run_ours(args, world, rank, local):
         "kv_append_gbs": append_bytes(wl) / (app_ms * 1e-3) / 1e9,
         "roofline": roof,
         "e2e": e2e,
-        "gpu_launches": 4 * args.steps,
+        # per step: the append (one kernel up to 2047 agents, else schedule + append), schedule + attention
+        "gpu_launches": (3 if wl.B <= 2047 else 4) * args.steps,
         "clocks": clk,
     }
     if per_agent is not None:

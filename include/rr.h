@@ -83,6 +83,12 @@ typedef struct rr_dims {
  * checks this on the host); pages shared between agents (a common system
  * prompt) are only ever read.  A page id outside the pool is skipped and
  * recorded as RR_ERR_OOB in the device error word.
+ *
+ * For a batch of at most 2047 agents the call is a single kernel that checks
+ * the lengths and takes their prefix sums itself (it uses no workspace); a
+ * larger batch runs the device-side schedule first, in the workspace.  Either
+ * way, lengths inconsistent with total_tokens (or a negative length, or one
+ * past the page table) write nothing and record RR_ERR_LENS.
  */
 int rr_kv_append(const void* k_new, const void* v_new, void* k_pool, void* v_pool, const int32_t* page_table,
                  const int32_t* prefix_lens, const int32_t* suffix_lens, const rr_dims* dims,
@@ -116,7 +122,7 @@ int rr_extend_attention(const void* q, const void* k_pool, const void* v_pool, c
  * rr_extend_step -- the whole extend step of Sec. 2 in one attention launch:
  * the same results as rr_kv_append followed by rr_extend_attention on the
  * same stream (the pools receive the suffix K/V bit for bit, and `out` is
- * bit-identical), with two kernels launched instead of four.
+ * bit-identical), with two kernels launched instead of three.
  *
  * The kernel first writes every suffix row of k_new / v_new [T][Hkv][D] into
  * the pool slots page_table assigns to it, with all its threads; then every
