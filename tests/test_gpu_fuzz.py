@@ -1,5 +1,5 @@
-"""Seeded random batches through the append, the extend attention, the one-launch step and decode, against the
-fp64 oracle.
+"""Seeded random batches through the append, the extend attention, the one-launch step and decode, plain and
+with a rotary table, against the fp64 oracle.
 
 Each case draws its own shape -- head dim 64 or 128, 1-8 KV heads, GQA group 1-16, page size 8-128 -- and a
 batch of 1-9 agents whose cached prefixes may be empty, end mid-page or run to a few thousand keys, and whose
@@ -105,3 +105,38 @@ def test_random_batch(rr, case):
         refd = oracle.decode_attention(qd_bits, kp, vp, wl.page_table, L.astype(np.int32),
                                        scale=1.0 / math.sqrt(wl.D))
         check_close(to_f64(outd), refd, f"{case_id(case)} decode")
+
+
+BASE = 500000.0
+
+
+@pytest.mark.parametrize("case", CASES[::2], ids=[case_id(c) for c in CASES[::2]])
+def test_random_batch_rotary(rr, case):
+    """The same batches with q and k_new taken un-rotated (rotary table, base 5e5): the rotated append (V bit-exact;
+    K is checked against its error bound in the rotary tests) and attention against the oracle's rotation, and
+    the one-launch rotary step bit-identical to the two calls."""
+    import torch
+    wl = synth.custom(case["name"], case["B"], case["Hq"], case["Hkv"], case["D"], case["P"], case["S"],
+                      ps=case["ps"], seed=case["seed"])
+    host = synth.cpu_tensors(wl)
+    g = synth.gpu_tensors(wl, "cuda")
+    g2 = {k: v.clone() for k, v in g.items()}
+    table = rr.rope_table(int((wl.prefix_lens.astype(np.int64) + wl.suffix_lens).max()) + 1, wl.D, BASE)
+    rr.kv_append(g["k_new"], g["v_new"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                 g["suffix_lens"], rope=table)
+    out = rr.extend_attention(g["q"], g["k_pool"], g["v_pool"], g["page_table"], g["prefix_lens"],
+                              g["suffix_lens"], rope=table)
+    torch.cuda.synchronize()
+    assert rr.device_error() == 0, rr.last_error()
+    kp, vp = oracle.kv_append_rope(host["k_new"], host["v_new"], host["k_pool"], host["v_pool"], wl.page_table,
+                                   wl.prefix_lens, wl.suffix_lens, BASE)
+    np.testing.assert_array_equal(bf16_bits(g["v_pool"]), vp)
+    ref = oracle.extend_attention_rope(host["q"], kp, vp, wl.page_table, wl.prefix_lens, wl.suffix_lens, BASE,
+                                       scale=1.0 / math.sqrt(wl.D))
+    check_close(to_f64(out), ref, f"{case_id(case)} rotary extend")
+    out2 = rr.extend_step(g2["q"], g2["k_new"], g2["v_new"], g2["k_pool"], g2["v_pool"], g2["page_table"],
+                          g2["prefix_lens"], g2["suffix_lens"], rope=table)
+    torch.cuda.synchronize()
+    assert rr.device_error() == 0, rr.last_error()
+    np.testing.assert_array_equal(bf16_bits(g2["k_pool"]), bf16_bits(g["k_pool"]))
+    np.testing.assert_array_equal(bf16_bits(out2), bf16_bits(out))
