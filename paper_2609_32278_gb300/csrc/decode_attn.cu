@@ -18,7 +18,7 @@
 // S^T and O^T live in TMEM (lane = key, resp. lane = head dimension; column =
 // head); P^T is written by the softmax threads to shared memory.
 //
-// Roles (one persistent CTA per SM, 6 warps):
+// Roles (one persistent CTA per SM, 7 warps):
 //   * warps 0-3, softmax and epilogue: thread t owns key t of the tile (TMEM
 //     lane t of S^T).  Per head: mask keys past the agent's end, the tile max
 //     (warp shuffles, then the four warps' maxima through shared memory), a
@@ -27,10 +27,11 @@
 //     bf16, and a per-thread partial weight sum.  At the end of a work item
 //     thread t owns output dimension t: O^T row t / l, stored as bf16 (or the
 //     fp32 partial of a split item, merged by the combine kernel).
-//   * warp 4, TMA producer: Q^T (one 3-D box of G rows per 64-column chunk),
-//     then per 128-key tile one 2-D box per page and chunk for K and for V (the
-//     page gather), into a ring of NS stages; slots of the agent's last page
-//     past its end are cleared in shared memory before the MMA may read V.
+//   * warps 4 and 6, TMA producers, taking the 128-key tiles in turn: per tile
+//     one 2-D box per page and chunk for K and for V (the page gather), into a
+//     ring of NS stages; slots of the agent's last page past its end are
+//     cleared in shared memory before the MMA may read V.  Warp 4 also loads
+//     Q^T (one 3-D box of G rows per 64-column chunk).
 //   * warp 5, MMA issuer (one thread): S^T(t) into one of two TMEM buffers,
 //     then O^T += V(t-1)^T P^T(t-1), so the scores of tile t are computed while
 //     the softmax works on tile t-1.
@@ -55,8 +56,12 @@ namespace rr {
 
 namespace {
 
-constexpr int kDecThreads = 192;       // warps 0-3 softmax / epilogue, 4 producer, 5 MMA
-constexpr int kDecWarpProducer = 4;
+// TMA producer warps: warp 4, then 6, 7, ...  One warp issuing every page box of K and V (32 boxes per tile at
+// 16-token pages; a warp issues its lanes' boxes one after another) streamed c2_decode at 5.69 TB/s; two warps
+// taking the tiles in turn, 6.25 TB/s; three, 6.26 TB/s.
+constexpr int kDecProducers = 2;
+constexpr int kDecThreads = 32 * (6 + kDecProducers - 1);  // warps 0-3 softmax / epilogue, 5 MMA, the rest producers
+constexpr int kDecWarpProducer = 4;     // Q, and the K / V tiles the first producer takes
 constexpr int kDecWarpMMA = 5;
 constexpr int kHeadCols = 16;          // N of both MMAs: the G heads of a KV head, padded
 constexpr uint32_t kDecTmemCols = 64;  // S^T buffers at columns 0 and 16, O^T at 32
@@ -82,7 +87,8 @@ struct DecCfg {
     static constexpr int kOFinal = kPEmpty + 2, kOEmpty = kOFinal + 1, kXch = kOEmpty + 1, kDrain = kXch + 1;
     static constexpr int kDone = kDrain + 1;
     static constexpr int kQRot = kDone + 1;  // rotary q: the item's Q^T rows rotated in shared memory
-    static constexpr int kNumBars = kQRot + 1;
+    static constexpr int kVTmp2 = kQRot + 1;  // the other producers' side barriers for a partly owned last page
+    static constexpr int kNumBars = kVTmp2 + kDecProducers - 1;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // u32 TMEM base, i32 abort flag
     static constexpr int kSmemBytes = kOffMisc + 16 + 1024;  // + slack to align the base to 1 KiB
     static_assert(kStageBytes % 1024 == 0 && kOffQ % 1024 == 0 && kOffP % 1024 == 0,
@@ -222,6 +228,10 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
     using C = DecCfg<D, NS>;
     static_assert(!(kRope && kGroup), "shared-prefix items take rotated queries only");
     static_assert(G >= 1 && G <= kHeadCols, "one KV head's query heads must fit the 16 MMA columns");
+    // A producer waits for a stage's previous phase by parity, which is exact only while the barrier can be at
+    // most one phase behind: a producer's own previous tile (kDecProducers tiles back) bounds its lead to that
+    // only if kDecProducers <= NS.
+    static_assert(kDecProducers >= 1 && kDecProducers <= NS, "more producers than stages");
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const uint32_t sb = ptx::smem_u32(smem);
@@ -245,6 +255,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
             ptx::mbar_init(bar(C::kKVEmpty + s), 1);
         }
         ptx::mbar_init(bar(C::kVTmp), 1);
+        for (int i = 0; i < kDecProducers - 1; ++i) ptx::mbar_init(bar(C::kVTmp2 + i), 1);
         for (int i = 0; i < 2; ++i) {
             ptx::mbar_init(bar(C::kSFull + i), 1);
             ptx::mbar_init(bar(C::kSEmpty + i), 4);   // one arrival per softmax warp
@@ -279,8 +290,14 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
     const int grid = gridDim.x, cta = blockIdx.x;
     const int page0 = kGroup ? 0 : a.page0;  // page-table column of the item range's first key
 
-    if (warp == kDecWarpProducer) {
-        // ------------------------------------------------------------ TMA producer
+    if (warp == kDecWarpProducer || warp > kDecWarpMMA) {
+        // ------------------------------------------------------------ TMA producers
+        // A tile of small pages is many TMA boxes (K and V: 32 at 16-token pages), and a warp issues its lanes'
+        // boxes one after another; one warp alone kept too few bytes in flight for HBM.  The producers take the
+        // tiles in turn (by the running tile count), each waiting for its own tiles' stages.
+        const bool first_warp = warp == kDecWarpProducer;
+        const uint32_t pi = first_warp ? 0u : (uint32_t)(warp - kDecWarpMMA);  // producer index
+        const uint32_t vtmp_bar = bar(first_warp ? C::kVTmp : C::kVTmp2 + (int)pi - 1);
         const int ppt = kBN / a.ps;  // pages per tile (<= 16)
         uint32_t gt = 0, item_i = 0, vtmp_phase = 0;
         int armed_q = -1, armed_vtmp = -1;  // copies in flight, for the abort drain
@@ -292,7 +309,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
             const DecItem it = dec_item<kGroup>(a, ui);
             const int b = it.b, g = it.g, kb = it.kb, ke = it.ke, L = it.L;
             const int last_page_end = ((L + a.ps - 1) / a.ps) * a.ps;
-            if (lane == 0) {
+            if (first_warp && lane == 0) {
                 if (item_i > 0) ok = dec_wait(bar(C::kQEmpty), (item_i - 1) & 1, ctl);
                 if (ok) {
                     // one box of 16 Q^T rows (group: group_agents agents x a.G heads; rows past the batch are
@@ -312,6 +329,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
             ok = __shfl_sync(0xffffffffu, ok, 0);
             if (!ok) break;
             for (int j = kb; j < ke; ++j, ++gt) {
+                if (gt % (uint32_t)kDecProducers != pi) continue;  // another producer's tile
                 const int s = (int)(gt % NS);
                 const uint32_t use = gt / NS;
                 int row = a.oob_row;  // page past the agent's keys: zero fill
@@ -340,7 +358,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
                 // V; if the agent's last page is only partly its own, land it on the side barrier, clear the
                 // slots past the agent's end, then release it
                 const bool clear_tail = (j == (L - 1) / kBN) && (last_page_end > L);
-                const uint32_t vbar = clear_tail ? bar(C::kVTmp) : bar(C::kVFull + s);
+                const uint32_t vbar = clear_tail ? vtmp_bar : bar(C::kVFull + s);
                 if (lane == 0) ptx::mbar_arrive_expect_tx(vbar, C::kTileBytes);
                 __syncwarp();
                 if (lane < ppt)
@@ -349,7 +367,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
                                          vbar);
                 if (clear_tail) {
                     armed_vtmp = (int)vtmp_phase;
-                    if (lane == 0) ok = dec_wait(bar(C::kVTmp), vtmp_phase, ctl);
+                    if (lane == 0) ok = dec_wait(vtmp_bar, vtmp_phase, ctl);
                     ok = __shfl_sync(0xffffffffu, ok, 0);
                     if (!ok) break;
                     armed_vtmp = -1;
@@ -371,7 +389,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
         }
         if (!ok && lane == 0) {  // abort: let every copy this warp started land before exit
             if (armed_q >= 0) dec_drain(bar(C::kQFull), (uint32_t)armed_q);
-            if (armed_vtmp >= 0) dec_drain(bar(C::kVTmp), (uint32_t)armed_vtmp);
+            if (armed_vtmp >= 0) dec_drain(vtmp_bar, (uint32_t)armed_vtmp);
             for (int s = 0; s < NS; ++s) {
                 if (armed_k >> s & 1u) dec_drain(bar(C::kKFull + s), par_k >> s & 1u);
                 if (armed_v >> s & 1u) dec_drain(bar(C::kVFull + s), par_v >> s & 1u);
