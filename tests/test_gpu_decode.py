@@ -68,6 +68,12 @@ CASES = [
     ("split_one_long_agent", 1, 8, 2, 128, [20000]),
     ("split_two_agents_d64", 2, 8, 2, 64, [9000, 3100]),
     ("split_g8_midpage", 1, 16, 2, 128, [12345]),
+    # every agent's last page partly its own, on tiles 0-7 of the agent and split into pieces of different
+    # lengths: a CTA's producer warps take its tiles in turn, so the tail tiles fall to both producers and
+    # both side barriers that hold a partly owned V page are used in one call
+    ("tails_alternate_producers", 8, 8, 2, 128, [128 * k + 5 + 2 * k for k in range(8)]),
+    ("tails_alternate_producers_d64", 7, 8, 2, 64, [128 * k + 9 for k in range(7)]),
+    ("tails_split_one_agent", 1, 8, 2, 128, [9 * 1024 + 7]),
 ]
 
 
