@@ -39,6 +39,7 @@ __device__ __forceinline__ int last_le(const int32_t* off, int n, long long x) {
 }
 
 constexpr int kAppendThreads = 256;
+constexpr int kAppendBlocksPerSM = 4;  // resident blocks per SM: at most 64 registers a thread
 constexpr int kCuSmem = 2048;  // agents whose suffix prefix sums a block stages in shared memory
 static_assert(kAppendSelfLensMaxB < kCuSmem, "the self-checking path keeps B + 1 prefix sums in shared memory");
 
@@ -46,7 +47,7 @@ static_assert(kAppendSelfLensMaxB < kCuSmem, "the self-checking path keeps B + 1
 // kCuSmem agents): each thread takes a contiguous run of agents, checks 0 <= P, 0 <= S, P + S <= the page
 // table's capacity, and the block scans the suffix lengths into s_cu[0..B]; the sum must equal T.  Every block
 // reaches the same verdict from the same lengths; block 0 reports a bad batch (RR_ERR_LENS) and no block writes.
-__device__ bool self_lens(const AppendArgs& a, int32_t* s_cu) {
+__device__ bool self_lens(const AppendArgs& a, int32_t* s_cu, int32_t* s_pfx) {
     __shared__ long long s_w[kAppendThreads / 32];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int B = a.B;
@@ -82,6 +83,7 @@ __device__ bool self_lens(const AppendArgs& a, int32_t* s_cu) {
     }
     for (int b = b0; b < b1; ++b) {
         s_cu[b] = (int32_t)off;
+        s_pfx[b] = a.prefix[b];
         off += a.suffix[b];
     }
     if (threadIdx.x == 0) s_cu[B] = (int32_t)total;
@@ -92,23 +94,29 @@ __device__ bool self_lens(const AppendArgs& a, int32_t* s_cu) {
 
 // kSelf: the lengths are checked and summed by the kernel itself (self_lens) instead of by the schedule kernel.
 template <bool kRope, bool kSelf>
-__global__ void __launch_bounds__(kAppendThreads) kv_append_kernel(const AppendArgs a) {
+__global__ void __launch_bounds__(kAppendThreads, kAppendBlocksPerSM) kv_append_kernel(const AppendArgs a) {
     __shared__ int32_t s_cu[kCuSmem];
-    // each token's agent is a binary search over the suffix prefix sums: from shared memory when they fit,
-    // so a token's copy does not wait behind log2(B) dependent global loads
+    __shared__ int32_t s_pfx[kCuSmem];
+    // each token's agent is a binary search over the suffix prefix sums, and its position needs the agent's
+    // prefix length: both from shared memory when they fit, so a token's copy does not wait behind dependent
+    // global loads
     bool cu_in_smem = true;
     if constexpr (kSelf) {
-        if (!self_lens(a, s_cu)) return;
+        if (!self_lens(a, s_cu, s_pfx)) return;
     } else {
         ptx::griddep_wait();  // the schedule kernel's output (launched as its dependent)
         if (*a.lens_ok == 0) return;
         cu_in_smem = a.B < kCuSmem;
         if (cu_in_smem) {
-            for (int i = threadIdx.x; i <= a.B; i += kAppendThreads) s_cu[i] = a.cu[i];
+            for (int i = threadIdx.x; i <= a.B; i += kAppendThreads) {
+                s_cu[i] = a.cu[i];
+                if (i < a.B) s_pfx[i] = a.prefix[i];
+            }
             __syncthreads();
         }
     }
     const int32_t* __restrict__ cu = cu_in_smem ? s_cu : a.cu;
+    const int32_t* __restrict__ pfx = cu_in_smem ? s_pfx : a.prefix;
     const int lane = threadIdx.x & 31;
     const long long warps = (long long)gridDim.x * (kAppendThreads / 32);
     const uint4* __restrict__ kn = a.k_new;
@@ -117,15 +125,47 @@ __global__ void __launch_bounds__(kAppendThreads) kv_append_kernel(const AppendA
     uint4* __restrict__ vp = a.v_pool;
     for (long long t = (long long)blockIdx.x * (kAppendThreads / 32) + (threadIdx.x >> 5); t < a.T; t += warps) {
         const int b = last_le(cu, a.B, t);
-        const long long pos = (long long)a.prefix[b] + (t - cu[b]);
-        const int page = a.page_table[(long long)b * a.max_pages + pos / a.ps];
-        if (page < 0 || (long long)page >= a.num_pages) {
-            if (lane == 0) atomicCAS(a.err, 0, RR_ERR_OOB);
-            continue;
-        }
+        const long long pos = (long long)pfx[b] + (t - cu[b]);
         const long long src = t * a.row16;
-        const long long dst = ((long long)page * a.ps + pos % a.ps) * a.row16;
-        if constexpr (kRope) {
+        if constexpr (!kRope) {
+            // 128 vectors of K and 128 of V at a time (the whole row up to Hkv * D = 1024), four of each per
+            // lane; the first ones are read before the page-table entry comes back, so the two loads' latencies
+            // overlap
+            long long dst = -1;
+            for (int c0 = 0; c0 < a.row16; c0 += 128) {
+                uint4 kx[4], vx[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int e = c0 + lane + 32 * i;
+                    if (e < a.row16) {
+                        kx[i] = __ldcs(kn + src + e);
+                        vx[i] = __ldcs(vn + src + e);
+                    }
+                }
+                if (c0 == 0) {
+                    const int page = a.page_table[(long long)b * a.max_pages + pos / a.ps];
+                    if (page < 0 || (long long)page >= a.num_pages) {
+                        if (lane == 0) atomicCAS(a.err, 0, RR_ERR_OOB);
+                        break;
+                    }
+                    dst = ((long long)page * a.ps + pos % a.ps) * a.row16;
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int e = c0 + lane + 32 * i;
+                    if (e < a.row16) {
+                        kp[dst + e] = kx[i];
+                        vp[dst + e] = vx[i];
+                    }
+                }
+            }
+        } else {
+            const int page = a.page_table[(long long)b * a.max_pages + pos / a.ps];
+            if (page < 0 || (long long)page >= a.num_pages) {
+                if (lane == 0) atomicCAS(a.err, 0, RR_ERR_OOB);
+                continue;
+            }
+            const long long dst = ((long long)page * a.ps + pos % a.ps) * a.row16;
             if (pos >= a.rope_max_pos) {  // no table row for this position: nothing written, reported
                 if (lane == 0) atomicCAS(a.err, 0, RR_ERR_LENS);
                 continue;
@@ -149,22 +189,6 @@ __global__ void __launch_bounds__(kAppendThreads) kv_append_kernel(const AppendA
                 kp[dst + lo] = k0;
                 kp[dst + hi] = k1;
             }
-            continue;
-        }
-        int e = lane;
-        for (; e + 96 < a.row16; e += 128) {  // four vectors of K and four of V in flight per lane
-            uint4 k0 = __ldcs(kn + src + e), k1 = __ldcs(kn + src + e + 32);
-            uint4 k2 = __ldcs(kn + src + e + 64), k3 = __ldcs(kn + src + e + 96);
-            uint4 v0 = __ldcs(vn + src + e), v1 = __ldcs(vn + src + e + 32);
-            uint4 v2 = __ldcs(vn + src + e + 64), v3 = __ldcs(vn + src + e + 96);
-            kp[dst + e] = k0; kp[dst + e + 32] = k1; kp[dst + e + 64] = k2; kp[dst + e + 96] = k3;
-            vp[dst + e] = v0; vp[dst + e + 32] = v1; vp[dst + e + 64] = v2; vp[dst + e + 96] = v3;
-        }
-        for (; e < a.row16; e += 32) {
-            uint4 k0 = __ldcs(kn + src + e);
-            uint4 v0 = __ldcs(vn + src + e);
-            kp[dst + e] = k0;
-            vp[dst + e] = v0;
         }
     }
 }
@@ -174,7 +198,9 @@ __global__ void __launch_bounds__(kAppendThreads) kv_append_kernel(const AppendA
 cudaError_t launch_kv_append(const AppendArgs& a, int sm_count, cudaStream_t st) {
     const long long warps_needed = a.T;
     long long blocks = (warps_needed + (kAppendThreads / 32) - 1) / (kAppendThreads / 32);
-    const long long cap = (long long)sm_count * 8;  // 8 resident blocks of 256 threads per SM
+    // two waves of resident blocks (a second-wave block starts as a first-wave one finishes): 2-7 % faster than
+    // a grid of one wave on the c2 / c5 / c3_rr appends
+    const long long cap = (long long)sm_count * kAppendBlocksPerSM * 2;
     if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
     if (a.self_lens) {  // an ordinary launch: it runs once the kernels before it on the stream have finished
