@@ -46,7 +46,7 @@ static_assert(kAppendSelfLensMaxB < kCuSmem, "the self-checking path keeps B + 1
 // The schedule kernel's length check and prefix sums, done by one block for itself (batches of fewer than
 // kCuSmem agents): each thread takes a contiguous run of agents, checks 0 <= P, 0 <= S, P + S <= the page
 // table's capacity, and the block scans the suffix lengths into s_cu[0..B]; the sum must equal T.  Every block
-// reaches the same verdict from the same lengths; block 0 reports a bad batch (RR_ERR_LENS) and no block writes.
+// reaches the same answer from the same lengths; block 0 reports a bad batch (RR_ERR_LENS) and no block writes.
 __device__ bool self_lens(const AppendArgs& a, int32_t* s_cu, int32_t* s_pfx) {
     __shared__ long long s_w[kAppendThreads / 32];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
