@@ -485,6 +485,8 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
     }
 
     // ================================================================ softmax / epilogue (warps 0-3)
+    // Pipeline waits are warp-uniform (__all_sync): after an abort a lane that saw its phase complete must not go
+    // on to a warp-collective tcgen05 instruction or shuffle while a lane of the same warp has left the loop.
     {
         const int t_in = threadIdx.x;  // key of the tile, and output dimension in the epilogue
         const uint32_t lane_bits = (uint32_t)(warp * 32) << 16;
@@ -502,7 +504,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
             const DecItem it = dec_item<kGroup>(a, ui);
             const int b = it.b, g = it.g, kb = it.kb, ke = it.ke, L = it.L;
             if constexpr (kRope) {  // rotate the item's Q^T rows once they have landed
-                if (!(ok = dec_wait(bar(C::kQFull), item_i & 1, ctl))) break;
+                if (!(ok = __all_sync(0xffffffffu, dec_wait(bar(C::kQFull), item_i & 1, ctl)))) break;
                 dec_rope_q<D, G>(smem + C::kOffQ, threadIdx.x, a.rope, a.rope_max_pos, L - 1, a.err);
                 ptx::fence_proxy_async_smem();  // generic-proxy writes -> the tensor core's reads
                 ptx::mbar_arrive(bar(C::kQRot));
@@ -512,7 +514,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
             for (int h = 0; h < G; ++h) { m[h] = -INFINITY; lp[h] = 0.f; }
             for (int j = kb; j < ke; ++j, ++gt) {
                 const int buf = (int)(gt & 1);
-                if (!(ok = dec_wait(bar(C::kSFull + buf), (gt >> 1) & 1, ctl))) break;
+                if (!(ok = __all_sync(0xffffffffu, dec_wait(bar(C::kSFull + buf), (gt >> 1) & 1, ctl)))) break;
                 ptx::tc_fence_after();
                 uint32_t sr[16];
                 tmem_ld16(tmem + lane_bits + (uint32_t)(buf * kHeadCols), sr);
@@ -543,7 +545,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
                 }
                 __syncwarp();
                 if (lane == 0) ptx::mbar_arrive(bar(C::kXch));
-                if (!(ok = dec_wait(bar(C::kXch), x_par, ctl))) break;
+                if (!(ok = __all_sync(0xffffffffu, dec_wait(bar(C::kXch), x_par, ctl)))) break;
                 x_par ^= 1u;
                 bool grow = false;
                 float f[G], p[G];
@@ -569,7 +571,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
                     lp[h] += p[h];
                 }
                 // P^T(gt) goes to buffer buf once O^T(gt-2) has read it
-                if (gt >= 2 && !(ok = dec_wait(bar(C::kPEmpty + buf), ((gt - 2) >> 1) & 1, ctl))) break;
+                if (gt >= 2 && !(ok = __all_sync(0xffffffffu, dec_wait(bar(C::kPEmpty + buf), ((gt - 2) >> 1) & 1, ctl)))) break;
                 const uint32_t pb = sb + C::kOffP + (uint32_t)(buf * C::kPBytes) + p_key_off;
                 {
                     float nb[G];
@@ -587,7 +589,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
                 // O^T holds V^T P^T of tiles < j once O^T(gt-1) has completed; bring it to the new max
                 // before O^T(gt) may start.  The max is the same in every thread, so is the branch.
                 if (grow) {
-                    if (!(ok = dec_wait(bar(C::kPEmpty + (int)((gt - 1) & 1)), ((gt - 1) >> 1) & 1, ctl))) break;
+                    if (!(ok = __all_sync(0xffffffffu, dec_wait(bar(C::kPEmpty + (int)((gt - 1) & 1)), ((gt - 1) >> 1) & 1, ctl)))) break;
                     ptx::tc_fence_after();
                     uint32_t o[16];
                     tmem_ld16(tmem + lane_bits + 2u * kHeadCols, o);
@@ -620,9 +622,9 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_attn_kernel(const __gri
             }
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(bar(C::kXch));
-            if (!(ok = dec_wait(bar(C::kXch), x_par, ctl))) break;
+            if (!(ok = __all_sync(0xffffffffu, dec_wait(bar(C::kXch), x_par, ctl)))) break;
             x_par ^= 1u;
-            if (!(ok = dec_wait(bar(C::kOFinal), item_i & 1, ctl))) break;
+            if (!(ok = __all_sync(0xffffffffu, dec_wait(bar(C::kOFinal), item_i & 1, ctl)))) break;
             ptx::tc_fence_after();
             uint32_t o[16];
             tmem_ld16(tmem + lane_bits + 2u * kHeadCols, o);

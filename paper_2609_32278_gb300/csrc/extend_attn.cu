@@ -697,6 +697,8 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
     return;
     }
     // ================================================================ softmax warpgroups (warps 0-7)
+    // Their pipeline waits are warp-uniform (__all_sync): after an abort a lane that saw its phase complete must
+    // not go on to a warp-collective tcgen05 instruction while a lane of the same warp has left the loop.
     ptx::setmaxnreg_inc<kRegsSoftmax>();
     {
         const int q = warp >> 2;                // Q tile of this warpgroup
@@ -727,7 +729,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             const int row_limit = min(P + tq0 + r / a.G, agent_len - 1);     // last key this row may see
             const int mask_from = (min(P + tq0, agent_len - 1) + 1) / kBN;  // earlier tiles: no masking
             if constexpr (kRope) {  // rotate this thread's row of Q tile q once the tile has landed
-                if (!(ok = wait_bar(bar(C::kQFull), q_phase, ctl))) break;
+                if (!(ok = __all_sync(0xffffffffu, wait_bar(bar(C::kQFull), q_phase, ctl)))) break;
                 q_phase ^= 1u;
                 const int tok = tq0 + r / a.G;
                 if (tok < a.suffix[b]) {  // rows past the agent's suffix are never stored
@@ -742,7 +744,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             }
             float m_run = -INFINITY, l_run = 0.f;
             for (int j = kb; j < ke; ++j) {
-                if (!(ok = wait_bar(bar(C::kSFull + q), s_phase, ctl))) break;
+                if (!(ok = __all_sync(0xffffffffu, wait_bar(bar(C::kSFull + q), s_phase, ctl)))) break;
                 s_phase ^= 1;
                 ptx::tc_fence_after();
                 // S row in two halves: the second half's TMEM load overlaps the first half's max.
@@ -849,7 +851,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
             }
             if (!ok) break;
             if constexpr (kCas == kCasShared) {
-                if (!(ok = wait_bar(bar(C::kOFinal + q), o_phase, ctl))) break;
+                if (!(ok = __all_sync(0xffffffffu, wait_bar(bar(C::kOFinal + q), o_phase, ctl)))) break;
                 o_phase ^= 1;
                 ptx::tc_fence_after();
                 // this row's unnormalised O and (max, sum) at (token, head), for the private pass to merge
@@ -880,7 +882,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                 const long long prow = (long long)(a.cu[b] + tok) * a.Hq + g * a.G + r % a.G;
                 const float4* so = reinterpret_cast<const float4*>(a.cas_o + prow * D);
                 const float2 ml = valid ? a.cas_ml[prow] : make_float2(-INFINITY, 0.f);  // in flight during the wait
-                if (!(ok = wait_bar(bar(C::kOFinal + q), o_phase, ctl))) break;
+                if (!(ok = __all_sync(0xffffffffu, wait_bar(bar(C::kOFinal + q), o_phase, ctl)))) break;
                 o_phase ^= 1;
                 ptx::tc_fence_after();
                 const float M = fmaxf(ml.x, m_run);  // m_run is finite: a row sees at least its own key here
@@ -923,7 +925,7 @@ __global__ void __launch_bounds__(kThreads, 1) extend_attn_kernel(const __grid_c
                 }
                 continue;
             }
-            if (!(ok = wait_bar(bar(C::kOFinal + q), o_phase, ctl))) break;
+            if (!(ok = __all_sync(0xffffffffu, wait_bar(bar(C::kOFinal + q), o_phase, ctl)))) break;
             o_phase ^= 1;
             ptx::tc_fence_after();
             const int slot = a.item_slot[ui];
